@@ -1,0 +1,68 @@
+"""Plant mistakes in the oracle (CPU only) and check that the pins catch each one.
+
+Each mutant is the oracle C source compiled with AIO_ORACLE_MUTANT=k:
+  1 dropped term, 2 transposed operand, 3 wrong sign, 4 wrong scale index,
+  5 dequantized weight rounded to bf16 before the product, 6 lost code sign.
+"""
+import struct
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from oracle import build as ob
+
+
+def _bf16_int(v):
+    return struct.unpack("<I", struct.pack("<f", float(v)))[0] >> 16
+
+
+def _exact(h):
+    h = int(h)
+    sign = -1 if h & 0x8000 else 1
+    e, m = (h >> 7) & 0xFF, h & 0x7F
+    return sign * (1 + Fraction(m, 128)) * Fraction(2) ** (e - 127) if e else sign * Fraction(m, 128) * Fraction(2) ** -126
+
+
+def pins_hold(o: oracle.Oracle) -> bool:
+    rng = np.random.default_rng(0)
+    # brute force, integer-valued bf16
+    xi = rng.integers(-8, 9, size=(2, 12))
+    wi = rng.integers(-8, 9, size=(5, 12))
+    to = np.vectorize(_bf16_int, otypes=[np.uint16])
+    y = o.linear_bf16(to(xi), to(wi))
+    if not np.array_equal(y, xi @ wi.T):
+        return False
+    # one-hot column selection with N != K
+    K, N = 9, 4
+    W = synth.normal_bf16(synth.key(1), 1.0, N * K).reshape(N, K)
+    for k in range(K):
+        x = np.zeros((1, K), np.uint16)
+        x[0, k] = _bf16_int(1)
+        if [Fraction(v) for v in o.linear_bf16(x, W)[0]] != [_exact(W[n, k]) for n in range(N)]:
+            return False
+    # int8: one-hot with distinct scales, and exact dequant of known codes
+    q = rng.integers(-127, 128, size=(N, K)).astype(np.int8)
+    s = synth.uniform_bf16(synth.key(2), 1e-3, 1e-2, N)
+    for k in range(K):
+        x = np.zeros((1, K), np.uint16)
+        x[0, k] = _bf16_int(1)
+        y = o.linear_i8(x, q, s)
+        if any(Fraction(y[0, n]) != _exact(s[n]) * int(q[n, k]) for n in range(N)):
+            return False
+    x = np.array([[_bf16_int(1)]], np.uint16)
+    if o.linear_i8(x, np.array([[127]], np.int8), np.array([0x3BA4], np.uint16))[0, 0] != 0.6356201171875:
+        return False
+    return True
+
+
+def test_shipped_oracle_passes_pins():
+    assert pins_hold(oracle.Oracle(oracle.load()))
+
+
+@pytest.mark.parametrize("mutant", [1, 2, 3, 4, 5, 6])
+def test_mutant_is_caught(tmp_path, mutant):
+    path = ob.build(out=str(tmp_path / f"libaio_oracle_m{mutant}.so"), mutant=mutant)
+    assert not pins_hold(oracle.Oracle(oracle.load(path)))
