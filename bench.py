@@ -1,0 +1,419 @@
+#!/usr/bin/env python
+"""Decode-step weight-streaming benchmark (A-IO, arxiv 2604.09752): weight-stream GB/s and
+equivalent decode tokens/s on GB300.
+
+A step is one pass of every projection of a decoder (Sec. 3.1: each generated token streams all
+weights from HBM): 4 projections per layer plus the lm_head, replayed as one CUDA graph with
+programmatic dependent launch.  Default workload: the 7B-class decode step at M=1 in bf16
+(32 layers, 129 projections, 13.21 GB of weights per token), synthetic seeded weights.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  Multi-GPU: one process per GPU (torchrun); each rank runs an
+independent replica (the path is replicated, not sharded) and ``value`` sums all ranks' bytes
+over the slowest rank's time.  ``--impl reference`` times the fp64 CPU oracle on a bounded
+sample of the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import datetime as _dt
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "weight-stream GB/s (% of GB300 HBM peak); equivalent decode tokens/s at M=1"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def workload_by_name(name):
+    from synth import workloads as swl
+    if name in swl.WORKLOADS:
+        return swl.WORKLOADS[name]
+    if name.startswith("7b-pld-"):
+        _, _, wt, m = name.split("-")
+        return swl.pld_workload(int(m[1:]), wt)
+    raise SystemExit(f"unknown workload {name}; choose from {sorted(swl.WORKLOADS)} or 7b-pld-<bf16|int8>-M<m>")
+
+
+def measured_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs: torch copy, read+write)"
+    return FALLBACK_HBM_GBS, "fallback (no MEASURED_PEAKS.json)"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("aio_gemv.cu", "aio_internal.h"):
+        h.update(open(os.path.join(ROOT, "paper_2604_09752_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(workload_name, launches_per_step):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current kernel."""
+    p = os.path.join(ROOT, "profiles", "gemv_traffic.txt")
+    if not os.path.exists(p):
+        return None, "no committed ncu traffic summary"
+    kv = {}
+    for line in open(p):
+        line = line.strip()
+        if line and not line.startswith("#") and " " in line:
+            k, v = line.split(None, 1)
+            kv[k] = v
+    if kv.get("kernel_src_sha") != kernel_source_hash():
+        return None, "kernel changed since the committed ncu capture"
+    if kv.get("workload") != workload_name or "dram_bytes_per_step" not in kv:
+        return None, f"committed capture is for workload {kv.get('workload')}"
+    return float(kv["dram_bytes_per_step"]) / launches_per_step, kv.get("note", "ncu dram__bytes_read+write")
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms in the background."""
+
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={index}", f"--query-gpu={self.FIELDS}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.p = None
+
+    def stop(self, t0, t1):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "note": "nvidia-smi unavailable"}
+        self.p.terminate()
+        self.p.wait()
+        self.f.seek(0)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, smax, reasons, n_all = [], [], set(), 0
+        for line in self.f.read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 10:
+                continue
+            n_all += 1
+            try:
+                ts = _dt.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+            except ValueError:
+                continue
+            if not (t0 - 0.25 <= ts <= t1 + 0.25):
+                continue
+            try:
+                sm.append(float(parts[2]))
+                smax.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[6:10]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        os.unlink(self.f.name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ---------------------------------------------------------------------------------------------
+def oracle_sample(wl, seed, frac):
+    """The first ceil(frac*N) rows of every projection, regenerated on the host: [(x, W, s)], bytes."""
+    from synth import workloads as swl
+    items, nbytes = [], 0
+    for p in wl.projs:
+        rows = max(1, math.ceil(frac * p.N))
+        x = swl.gen_x(seed, wl, p, wl.M).reshape(wl.M, p.K)
+        if wl.wtype == "int8":
+            W = swl.gen_codes(seed, wl, p, 0, rows).reshape(rows, p.K)
+            s = swl.gen_scales(seed, wl, p, 0, rows)
+            nbytes += rows * p.K + 2 * rows
+        else:
+            W = swl.gen_w_bf16(seed, wl, p, 0, rows).reshape(rows, p.K)
+            s = None
+            nbytes += rows * p.K * 2
+        items.append((x, W, s))
+    return items, nbytes
+
+
+def time_oracle(items):
+    """Seconds for one pass of the fp64 oracle over a sample, and the threads it used."""
+    import oracle
+    t0 = time.perf_counter()
+    for x, W, s in items:
+        if s is None:
+            oracle.linear_bf16(x, W)
+        else:
+            oracle.linear_i8(x, W, s)
+    return time.perf_counter() - t0, oracle.threads()
+
+
+def cpu_oracle_sample(wl, seed, frac):
+    items, nbytes = oracle_sample(wl, seed, frac)
+    dt, cores = time_oracle(items)
+    return dt, nbytes, cores
+
+
+def run_reference(args, wl):
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return 0
+    # calibrate: a 1/512 sample, then size each step to about 1 s of oracle work
+    dt0, b0, cores = cpu_oracle_sample(wl, args.seed, 1.0 / 512)
+    per_byte = dt0 / b0
+    full = wl.weight_bytes()
+    budget_s = max(0.2, min(2.0, 150.0 / max(1, args.steps + args.warmup)))
+    frac = min(1.0, budget_s / (per_byte * full))
+    items, nbytes = oracle_sample(wl, args.seed, frac)
+    dts = []
+    for i in range(args.warmup + args.steps):
+        dt, cores = time_oracle(items)
+        if i >= args.warmup:
+            dts.append(dt)
+    t = sum(dts) / len(dts)
+    gbs = nbytes / t / 1e9
+    sample = f"first {frac:.4%} of the rows of all {len(wl.projs)} projections ({nbytes} weight bytes) per step"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(gbs, 3), "unit": "GB/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t * 1000, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "M": wl.M, "wtype": wl.wtype, "projections": len(wl.projs),
+                   "weight_bytes_per_token": full},
+        "tokens_per_s_equivalent": round(gbs * 1e9 / full, 4),
+        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------------------------
+def run_ours(args, wl):
+    import torch
+    world, rank, local = dist_setup()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU (libaio is sm_103a only); no CPU fallback")
+    torch.cuda.set_device(local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        pg = dist
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+
+    M = wl.M
+    t_setup = time.perf_counter()
+    dw = DeviceWorkload(wl, seed=args.seed + rank, max_M=M)
+    x_host = dw.fill_x(M)
+    setup_s = time.perf_counter() - t_setup
+    stream = torch.cuda.Stream()
+    sh = stream.cuda_stream
+    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL
+    step = dw.step_handle(M, flags)
+    n_kernels = aio.aio_decode_step_kernels(step)
+    wbytes = dw.weight_bytes()
+
+    def barrier():
+        if pg is not None:
+            pg.barrier()
+
+    def max_over_ranks(v):
+        if pg is None:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        return float(t.item())
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            aio.aio_decode_step(step, sh)
+    torch.cuda.synchronize()
+    assert aio.aio_decode_step_check(step) == 0
+
+    # ---- device-resident timed region
+    clocks = ClockSampler(local)
+    time.sleep(0.4)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    w0 = time.time()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        aio.aio_decode_step(step, sh)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    w1 = time.time()
+    barrier()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    clk = clocks.stop(w0, w1)
+    ms_max = max_over_ranks(ms)
+    assert aio.aio_decode_step_check(step) == 0
+
+    # ---- end to end: pinned host x -> device, step, device y -> pinned host, every step
+    y_host = torch.empty(dw.y_arena.numel(), dtype=torch.uint8, pin_memory=True)
+    for _ in range(3):
+        with torch.cuda.stream(stream):
+            dw.x_arena.copy_(x_host, non_blocking=True)
+            aio.aio_decode_step(step, sh)
+            y_host.copy_(dw.y_arena, non_blocking=True)
+    torch.cuda.synchronize()
+    e_steps = max(10, args.steps // 4)
+    barrier()
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(e_steps):
+            dw.x_arena.copy_(x_host, non_blocking=True)
+            aio.aio_decode_step(step, sh)
+            y_host.copy_(dw.y_arena, non_blocking=True)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    e_ms = max_over_ranks(ev0.elapsed_time(ev1) / e_steps)
+
+    # ---- largest projection alone (standalone kernel, same stream)
+    big = max(range(len(dw.bufs)), key=lambda i: dw.bufs[i].proj.N * dw.bufs[i].proj.K)
+    bp = dw.bufs[big].proj
+    with torch.cuda.stream(stream):
+        for _ in range(5):
+            dw.run_proj(big, M, sh)
+    reps = 50
+    ev0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            dw.run_proj(big, M, sh)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    big_ms = ev0.elapsed_time(ev1) / reps
+    esize = 1 if dw.i8 else 2
+    big_bytes = bp.N * bp.K * esize + (2 * bp.N if dw.i8 else 0)
+
+    # ---- read ceiling of the same bulk-copy ring (4 GiB, well above L2)
+    pbuf = torch.empty(4 << 30, dtype=torch.uint8, device="cuda")
+    pout = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for _ in range(3):
+        aio.aio_probe_read(pbuf.data_ptr(), pbuf.numel(), pout.data_ptr(), sh)
+    ev0.record(stream)
+    for _ in range(10):
+        aio.aio_probe_read(pbuf.data_ptr(), pbuf.numel(), pout.data_ptr(), sh)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    probe_gbs = pbuf.numel() * 10 / (ev0.elapsed_time(ev1) / 1e3) / 1e9
+    del pbuf
+
+    peak, peak_src = measured_peak()
+    gbs_rank = wbytes / (ms / 1e3) / 1e9
+    value = world * wbytes / (ms_max / 1e3) / 1e9
+    tokens = world * 1000.0 / ms_max
+    e2e_gbs = world * wbytes / (e_ms / 1e3) / 1e9
+    traffic, traffic_note = committed_traffic(wl.name, n_kernels)
+
+    line = None
+    if rank == 0:
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            dt, nbytes, cores = cpu_oracle_sample(wl, args.seed, args.cpu_frac)
+            cpu = {"value": round(nbytes / dt / 1e9, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                   "sample": f"first {args.cpu_frac:.2%} of the rows of all {len(wl.projs)} projections "
+                             f"({nbytes} weight bytes, {dt:.2f} s of fp64 oracle work)"}
+        line = {
+            "metric": METRIC,
+            "value": round(value, 2),
+            "unit": "GB/s",
+            "n_gpus": world,
+            "steps": args.steps,
+            "warmup": args.warmup,
+            "ms_per_step": round(ms_max, 4),
+            "higher_is_better": True,
+            "scaling": "weak",
+            "vs_baseline": None,
+            "dtype": "int8" if dw.i8 else "bf16",
+            "data": "synthetic",
+            "config": {
+                "workload": wl.name,
+                "description": wl.description,
+                "M": M, "wtype": wl.wtype, "projections": len(dw.bufs),
+                "weight_bytes_per_token": wbytes,
+                "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                "l2": "inputs larger than L2 (every step streams all weights, >= 2.39 GB)",
+                "graph": "one CUDA graph per step, PDL between projections",
+            },
+            "tokens_per_s": round(tokens, 2),
+            "verified_tokens_per_s_upper_bound": round(tokens * M, 2),
+            "pct_of_measured_peak": round(100 * gbs_rank / peak, 2),
+            "pct_of_nominal_8tbs": round(100 * gbs_rank / NOMINAL_HBM_GBS, 2),
+            "roofline": {
+                "bound": "hbm",
+                "kernel": f"aio_gemv_kernel<M={M}, {'int8' if dw.i8 else 'bf16'}>",
+                "achieved": round(gbs_rank, 2),
+                "peak": peak,
+                "unit": "GB/s",
+                "frac": round(gbs_rank / peak, 4),
+                "traffic": traffic,
+                "traffic_note": traffic_note,
+                "peak_source": peak_src,
+                "algorithmic_bytes_per_launch": round(wbytes / n_kernels, 1),
+                "avg_launch_ms": round(ms / n_kernels, 5),
+                "launches_per_step": n_kernels,
+            },
+            "kernel_alone": {"projection": bp.name, "K": bp.K, "N": bp.N, "ms": round(big_ms, 4),
+                             "GB/s": round(big_bytes / (big_ms / 1e3) / 1e9, 2)},
+            "probe_read_gbs": round(probe_gbs, 1),
+            "e2e": {"value": round(e2e_gbs, 2), "unit": "GB/s", "ms_per_step": round(e_ms, 4),
+                    "h2d_bytes_per_step": int(dw.x_arena.numel()), "d2h_bytes_per_step": int(dw.y_arena.numel()),
+                    "path": "pinned host x -> aio_decode_step -> pinned host y, same stream"},
+            "gpu_launches": args.steps * n_kernels,
+            "clocks": clk,
+            "setup_s": round(setup_s, 1),
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    dw.close()
+    if pg is not None:
+        pg.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="7b-bf16")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--cpu-frac", type=float, default=0.125)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    wl = workload_by_name(args.workload)
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,197 @@
+/*
+ * aio.h -- C ABI of libaio: decode-step weight-streaming linear layers on GB300 (sm_103a).
+ *
+ * The computation (A-IO, arxiv 2604.09752): during autoregressive decoding every
+ * generated token fetches every weight of every linear layer from HBM, so decode is
+ * bound by HBM bandwidth (Sec. 2.1; Sec. 3.1).  Each projection computes
+ *
+ *     y[m, n] = sum_k x[m, k] * W[n, k]                         (y = x W^T)
+ *
+ * for M = 1 token row (plain decoding) or M = 2..8 rows (prompt-lookup verification,
+ * Sec. 4.2).  W8A16 storage-only quantization (Sec. 2.4; Sec. 6.2) stores W as int8
+ * codes q with one bf16 scale s[n] per output channel:
+ *
+ *     y[m, n] = s[n] * sum_k x[m, k] * q[n, k]
+ *
+ * Types and layouts (all row-major, all device pointers unless stated):
+ *   x  [M, K]  bf16 (IEEE bfloat16 bit patterns), row stride K elements
+ *   W  [N, K]  bf16, or int8 codes in [-127, 127] (-128 is also computed exactly)
+ *   s  [N]     bf16 scales (int8 weights only)
+ *   y  [M, N]  fp32, row stride N elements; fp32 accumulation
+ *
+ * Conventions shared by every entry point:
+ *   - Every call returns an aio_status; on failure aio_last_error() (thread-local)
+ *     holds a one-line description.  Argument errors are detected on the host
+ *     before anything is launched; no entry point traps on the device.
+ *   - Ownership: the caller owns every buffer it passes (x, W, scales, y, packed
+ *     weights).  The library owns only its handles, their small device workspaces
+ *     and captured graphs, and frees them in the matching *_destroy call.
+ *   - Asynchrony: run / pack / step calls enqueue work on the given stream (a
+ *     cudaStream_t passed as void*, NULL = legacy default stream) and return without
+ *     synchronising.  Buffers must stay valid until the stream has executed the work.
+ *   - Devices: a handle or step belongs to the device that was current when it was
+ *     created; using it while another device is current returns AIO_ERR_STATE.
+ *   - Device-side waits are bounded.  A wait that expires sets an error word that
+ *     aio_linear_check / aio_decode_step_check report as AIO_ERR_DEVICE_TIMEOUT.
+ */
+#ifndef AIO_H
+#define AIO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define AIO_ABI_VERSION 1
+
+typedef enum {
+    AIO_OK = 0,
+    AIO_ERR_INVALID_ARG = 1,     /* bad size, null pointer, M out of range, shape mismatch */
+    AIO_ERR_UNSUPPORTED = 2,     /* device is not sm_103 (the library is built for sm_103a only) */
+    AIO_ERR_ALIGNMENT = 3,       /* a pointer is not aligned as documented */
+    AIO_ERR_CUDA = 4,            /* a CUDA runtime call failed; see aio_last_error() */
+    AIO_ERR_OOM = 5,             /* workspace allocation failed */
+    AIO_ERR_STATE = 6,           /* wrong device current, or handle used after destroy */
+    AIO_ERR_DEVICE_TIMEOUT = 7   /* a bounded device-side wait expired (reported by *_check) */
+} aio_status;
+
+typedef enum {
+    AIO_W_BF16 = 0,              /* W is bf16 */
+    AIO_W_INT8_PERCHANNEL = 1    /* W is int8 codes, one bf16 scale per output channel */
+} aio_wtype;
+
+/* aio_linear_create flags */
+#define AIO_FLAG_ROWMAJOR   0x1u   /* aio_linear_run reads W as plain row-major [N, K] (no packing) */
+#define AIO_FLAG_NO_PDL     0x2u   /* launch without programmatic dependent launch */
+#define AIO_FLAG_TEST_STALL 0x100u /* TEST ONLY: the grid's last warp skips its first weight copy,
+                                      so its bounded wait (20 ms) expires and the run reports
+                                      AIO_ERR_DEVICE_TIMEOUT; outputs are then undefined */
+
+/* aio_decode_step_create flags */
+#define AIO_STEP_GRAPH 0x1u        /* capture the whole step into one CUDA graph (one launch per step) */
+#define AIO_STEP_PDL   0x2u        /* programmatic dependent launch between consecutive projections */
+
+/* Packed weight layout written by aio_linear_pack (a permutation of W, no padding):
+ * rows are grouped 8 at a time and each group is cut into tiles of 256 k-columns;
+ * tile (g, kt) starts at element 8*g*K + rows_g*256*kt, rows_g = min(8, N - 8g), and is
+ * the row-major block W[8g : 8g+rows_g, 256kt : 256kt+len], len = min(256, K - 256kt). */
+#define AIO_ROWS_PER_GROUP 8
+#define AIO_K_TILE 256
+
+typedef struct aio_linear* aio_linear_t;
+typedef struct aio_step* aio_step_t;
+
+/* One projection of a decode step (all device pointers, see the layouts above). */
+typedef struct {
+    aio_linear_t h;       /* shape and weight type */
+    const void* x;        /* [M, K] bf16 */
+    const void* W;        /* packed weights (or row-major if h was created with AIO_FLAG_ROWMAJOR) */
+    const void* scales;   /* [N] bf16 for int8 weights, NULL for bf16 */
+    float* y;             /* [M, N] fp32 */
+} aio_proj;
+
+/* ABI version of the loaded library (AIO_ABI_VERSION at build time). */
+int aio_abi_version(void);
+
+/* Static description of an error code; never NULL. */
+const char* aio_status_string(aio_status s);
+
+/* Detail of the last failure on the calling thread ("" if none). */
+const char* aio_last_error(void);
+
+/*
+ * Create a handle for one linear layer y = x W^T with W [N, K] (Sec. 2.1; Sec. 2.4 for int8).
+ *   out    receives the handle (set to NULL on failure)
+ *   K      16 <= K <= 1048576 and K % 16 == 0
+ *   N      1 <= N <= 16777216
+ *   wt     AIO_W_BF16 or AIO_W_INT8_PERCHANNEL
+ *   max_M  1..8: the largest number of token rows later passed to aio_linear_run
+ *   flags  AIO_FLAG_* bits
+ * Allocates a small device workspace (cross-CTA partial sums and counters, zeroed here)
+ * on the current device; synchronises that device.  Errors: INVALID_ARG, UNSUPPORTED,
+ * OOM, CUDA.
+ */
+aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int max_M, unsigned flags);
+
+/* Bytes of the packed weight buffer (N*K*elem_size) and of the scale buffer (2*N for int8, else 0). */
+aio_status aio_linear_packed_bytes(aio_linear_t h, size_t* w_bytes, size_t* scale_bytes);
+
+/* Launch geometry of aio_linear_run: CTAs, threads per CTA, dynamic shared memory bytes,
+ * and the number of weight tiles the grid streams.  Any pointer may be NULL. */
+aio_status aio_linear_launch_info(aio_linear_t h, int* grid, int* block, size_t* smem_bytes, long long* tiles);
+
+/*
+ * Pack row-major W [N, K] (bf16 or int8, device) into the tiled layout above (device,
+ * aio_linear_packed_bytes bytes, must not overlap W).  For int8, scales [N] bf16 are copied
+ * to scales_packed (both device, or both NULL for bf16).  All pointers 16-byte aligned.
+ * Asynchronous on stream.  Errors: INVALID_ARG, ALIGNMENT, STATE, CUDA.
+ */
+aio_status aio_linear_pack(aio_linear_t h, const void* W_rowmajor, const void* scales,
+                           void* W_packed, void* scales_packed, void* stream);
+
+/* Inverse of aio_linear_pack for the weights (used by tests): packed -> row-major [N, K]. */
+aio_status aio_linear_unpack(aio_linear_t h, const void* W_packed, void* W_rowmajor, void* stream);
+
+/*
+ * y = x W^T for M token rows (Sec. 2.1; int8 with per-channel scales, Sec. 2.4).
+ *   x       [M, K] bf16, 16-byte aligned
+ *   M       1 <= M <= max_M of the handle
+ *   K, N    must equal the handle's
+ *   W       packed weights (row-major if the handle has AIO_FLAG_ROWMAJOR), 16-byte aligned
+ *   scales  [N] bf16, 2-byte aligned, non-NULL exactly when the handle is int8
+ *   y       [M, N] fp32, 16-byte aligned; fully overwritten
+ * Uses the handle's workspace: runs of one handle must not overlap in time (issue them on
+ * one stream, or order the streams).  With PDL (default) the kernel may start streaming W
+ * while the previous kernel on the stream is still running; it reads x and writes y only
+ * after that kernel has completed.  Errors: INVALID_ARG, ALIGNMENT, STATE, CUDA.
+ */
+aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, const void* W,
+                          const void* scales, float* y, void* stream);
+
+/* Synchronise the device, then report the handle's device error word:
+ * AIO_OK, or AIO_ERR_DEVICE_TIMEOUT (code also stored in *device_error if non-NULL). */
+aio_status aio_linear_check(aio_linear_t h, int* device_error);
+
+/* Clear the handle's workspace counters and error word (needed only after a device error). */
+aio_status aio_linear_reset(aio_linear_t h);
+
+/* Free the handle and its workspace (synchronises the device). NULL is accepted. */
+aio_status aio_linear_destroy(aio_linear_t h);
+
+/*
+ * Build one decode step: the projections run in array order on one stream, projection i+1
+ * reading its x only after projection i has completed (Sec. 3.1: every weight of every layer is
+ * streamed once per token).  Pointer values are captured at creation: later calls rewrite the
+ * buffers' contents, never their addresses.  1 <= M <= every handle's max_M.  The step owns a
+ * private workspace per projection (so consecutive projections may overlap under PDL).
+ * flags: AIO_STEP_GRAPH and/or AIO_STEP_PDL.  Errors: INVALID_ARG, ALIGNMENT, STATE, OOM, CUDA.
+ */
+aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_projs, int M, unsigned flags);
+
+/* Enqueue one decode step on stream (one graph launch with AIO_STEP_GRAPH). */
+aio_status aio_decode_step(aio_step_t step, void* stream);
+
+/* Number of kernels one aio_decode_step launches. */
+aio_status aio_decode_step_kernels(aio_step_t step, int* n_kernels);
+
+/* Synchronise the device, then report the step's device error word (see aio_linear_check). */
+aio_status aio_decode_step_check(aio_step_t step, int* device_error);
+
+/* Free the step, its graph and its workspace (synchronises the device). NULL is accepted. */
+aio_status aio_decode_step_destroy(aio_step_t step);
+
+/*
+ * Read-bandwidth probe: streams `bytes` from buf (device, 16-byte aligned, bytes a multiple of
+ * 4096) through the same per-warp bulk-copy ring the linear kernels use, touching every chunk,
+ * and XORs one word per chunk into *out (device uint32).  Measures the practical HBM read
+ * ceiling for the roofline.  Asynchronous on stream.
+ */
+aio_status aio_probe_read(const void* buf, size_t bytes, unsigned* out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* AIO_H */

@@ -1,0 +1,185 @@
+"""Thin ctypes binding of libaio (include/aio.h): same names, argument marshalling only.
+
+Every computation runs in libaio's CUDA kernels.  Device buffers are passed as
+integer addresses (e.g. ``tensor.data_ptr()``) and streams as integer handles
+(``torch.cuda.current_stream().cuda_stream``).  A non-OK status raises AioError
+carrying the code and libaio's detail message.  There is no fallback: if
+libaio.so is missing, importing this module raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libaio.so")
+HEADER = os.path.join(os.path.dirname(_HERE), "include", "aio.h")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it with __graft_entry__.build() (nvcc, sm_103a)")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+# status codes and flags, read from the header so the binding cannot drift from it
+_hdr = open(HEADER).read() if os.path.exists(HEADER) else ""
+AIO_OK = 0
+AIO_ERR_INVALID_ARG = 1
+AIO_ERR_UNSUPPORTED = 2
+AIO_ERR_ALIGNMENT = 3
+AIO_ERR_CUDA = 4
+AIO_ERR_OOM = 5
+AIO_ERR_STATE = 6
+AIO_ERR_DEVICE_TIMEOUT = 7
+AIO_W_BF16 = 0
+AIO_W_INT8_PERCHANNEL = 1
+AIO_FLAG_ROWMAJOR = 0x1
+AIO_FLAG_NO_PDL = 0x2
+AIO_FLAG_TEST_STALL = 0x100
+AIO_STEP_GRAPH = 0x1
+AIO_STEP_PDL = 0x2
+AIO_ROWS_PER_GROUP = 8
+AIO_K_TILE = 256
+for _name, _val in re.findall(r"#define\s+(AIO_\w+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", _hdr):
+    if _name in globals() and globals()[_name] != int(_val, 0):
+        raise ImportError(f"binding constant {_name} disagrees with include/aio.h")
+
+
+class AioError(RuntimeError):
+    def __init__(self, status: int, func: str):
+        self.status = status
+        detail = _lib.aio_last_error().decode(errors="replace")
+        name = _lib.aio_status_string(status).decode()
+        super().__init__(f"{func}: {name}: {detail}")
+
+
+class aio_proj(ctypes.Structure):
+    _fields_ = [("h", ctypes.c_void_p), ("x", ctypes.c_void_p), ("W", ctypes.c_void_p),
+                ("scales", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
+_vp, _int, _u = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint
+_sz, _ll = ctypes.c_size_t, ctypes.c_longlong
+_SIGS = {
+    "aio_abi_version": (_int, []),
+    "aio_status_string": (ctypes.c_char_p, [_int]),
+    "aio_last_error": (ctypes.c_char_p, []),
+    "aio_linear_create": (_int, [ctypes.POINTER(_vp), _int, _int, _int, _int, _u]),
+    "aio_linear_packed_bytes": (_int, [_vp, ctypes.POINTER(_sz), ctypes.POINTER(_sz)]),
+    "aio_linear_launch_info": (_int, [_vp, ctypes.POINTER(_int), ctypes.POINTER(_int), ctypes.POINTER(_sz),
+                                      ctypes.POINTER(_ll)]),
+    "aio_linear_pack": (_int, [_vp, _vp, _vp, _vp, _vp, _vp]),
+    "aio_linear_unpack": (_int, [_vp, _vp, _vp, _vp]),
+    "aio_linear_run": (_int, [_vp, _vp, _int, _int, _int, _vp, _vp, _vp, _vp]),
+    "aio_linear_check": (_int, [_vp, ctypes.POINTER(_int)]),
+    "aio_linear_reset": (_int, [_vp]),
+    "aio_linear_destroy": (_int, [_vp]),
+    "aio_decode_step_create": (_int, [ctypes.POINTER(_vp), ctypes.POINTER(aio_proj), _int, _int, _u]),
+    "aio_decode_step": (_int, [_vp, _vp]),
+    "aio_decode_step_kernels": (_int, [_vp, ctypes.POINTER(_int)]),
+    "aio_decode_step_check": (_int, [_vp, ctypes.POINTER(_int)]),
+    "aio_decode_step_destroy": (_int, [_vp]),
+    "aio_probe_read": (_int, [_vp, _sz, _vp, _vp]),
+}
+for _f, (_res, _args) in _SIGS.items():
+    _fn = getattr(_lib, _f)
+    _fn.restype = _res
+    _fn.argtypes = _args
+
+
+def lib():
+    return _lib
+
+
+def _check(status: int, func: str):
+    if status != AIO_OK:
+        raise AioError(status, func)
+
+
+def aio_abi_version() -> int:
+    return _lib.aio_abi_version()
+
+
+def aio_status_string(s: int) -> str:
+    return _lib.aio_status_string(s).decode()
+
+
+def aio_last_error() -> str:
+    return _lib.aio_last_error().decode(errors="replace")
+
+
+def aio_linear_create(K: int, N: int, wt: int, max_M: int, flags: int = 0) -> int:
+    h = _vp()
+    _check(_lib.aio_linear_create(ctypes.byref(h), K, N, wt, max_M, flags), "aio_linear_create")
+    return h.value
+
+
+def aio_linear_packed_bytes(h: int):
+    w, s = _sz(), _sz()
+    _check(_lib.aio_linear_packed_bytes(h, ctypes.byref(w), ctypes.byref(s)), "aio_linear_packed_bytes")
+    return w.value, s.value
+
+
+def aio_linear_launch_info(h: int):
+    g, b, sm, t = _int(), _int(), _sz(), _ll()
+    _check(_lib.aio_linear_launch_info(h, ctypes.byref(g), ctypes.byref(b), ctypes.byref(sm), ctypes.byref(t)),
+           "aio_linear_launch_info")
+    return {"grid": g.value, "block": b.value, "smem_bytes": sm.value, "tiles": t.value}
+
+
+def aio_linear_pack(h: int, W_rowmajor: int, scales, W_packed: int, scales_packed, stream: int = 0):
+    _check(_lib.aio_linear_pack(h, W_rowmajor, scales, W_packed, scales_packed, stream), "aio_linear_pack")
+
+
+def aio_linear_unpack(h: int, W_packed: int, W_rowmajor: int, stream: int = 0):
+    _check(_lib.aio_linear_unpack(h, W_packed, W_rowmajor, stream), "aio_linear_unpack")
+
+
+def aio_linear_run(h: int, x: int, M: int, K: int, N: int, W: int, scales, y: int, stream: int = 0):
+    _check(_lib.aio_linear_run(h, x, M, K, N, W, scales, y, stream), "aio_linear_run")
+
+
+def aio_linear_check(h: int) -> int:
+    e = _int()
+    _check(_lib.aio_linear_check(h, ctypes.byref(e)), "aio_linear_check")
+    return e.value
+
+
+def aio_linear_reset(h: int):
+    _check(_lib.aio_linear_reset(h), "aio_linear_reset")
+
+
+def aio_linear_destroy(h: int):
+    _check(_lib.aio_linear_destroy(h), "aio_linear_destroy")
+
+
+def aio_decode_step_create(projs, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP_PDL) -> int:
+    """projs: sequence of (h, x, W, scales, y) integer addresses (scales may be None)."""
+    arr = (aio_proj * len(projs))(*[aio_proj(*p) for p in projs])
+    s = _vp()
+    _check(_lib.aio_decode_step_create(ctypes.byref(s), arr, len(projs), M, flags), "aio_decode_step_create")
+    return s.value
+
+
+def aio_decode_step(step: int, stream: int = 0):
+    _check(_lib.aio_decode_step(step, stream), "aio_decode_step")
+
+
+def aio_decode_step_kernels(step: int) -> int:
+    n = _int()
+    _check(_lib.aio_decode_step_kernels(step, ctypes.byref(n)), "aio_decode_step_kernels")
+    return n.value
+
+
+def aio_decode_step_check(step: int) -> int:
+    e = _int()
+    _check(_lib.aio_decode_step_check(step, ctypes.byref(e)), "aio_decode_step_check")
+    return e.value
+
+
+def aio_decode_step_destroy(step: int):
+    _check(_lib.aio_decode_step_destroy(step), "aio_decode_step_destroy")
+
+
+def aio_probe_read(buf: int, nbytes: int, out: int, stream: int = 0):
+    _check(_lib.aio_probe_read(buf, nbytes, out, stream), "aio_probe_read")

@@ -1,0 +1,519 @@
+// aio_api.cu -- the C ABI (include/aio.h): argument validation, handles and their device
+// workspaces, kernel launches, and the decode step captured as one CUDA graph.
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <vector>
+
+#include "aio.h"
+#include "aio_internal.h"
+
+namespace {
+
+constexpr uint32_t kLinearMagic = 0xA10113EAu;
+constexpr uint32_t kStepMagic = 0xA1057E90u;
+constexpr unsigned kCreateFlags = AIO_FLAG_ROWMAJOR | AIO_FLAG_NO_PDL | AIO_FLAG_TEST_STALL;
+constexpr unsigned kStepFlags = AIO_STEP_GRAPH | AIO_STEP_PDL;
+constexpr unsigned long long kWaitLimitNs = 1000000000ull;      // 1 s: a healthy wait takes microseconds
+constexpr unsigned long long kTestWaitLimitNs = 20000000ull;    // 20 ms for AIO_FLAG_TEST_STALL
+
+thread_local char g_last_error[512] = "";
+
+aio_status fail(aio_status s, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+#define AIO_CUDA(expr)                                                                             \
+    do {                                                                                           \
+        cudaError_t e_ = (expr);                                                                   \
+        if (e_ != cudaSuccess) return fail(AIO_ERR_CUDA, "%s: %s", #expr, cudaGetErrorString(e_)); \
+    } while (0)
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+bool test_alloc_failure() {
+    const char* v = getenv("AIO_TEST_FAIL_ALLOC");
+    return v && v[0] == '1';
+}
+
+size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Device checks and one-time kernel attributes per device.
+std::mutex g_prep_mu;
+bool g_prepared[64] = {};
+
+aio_status current_device(int* dev, int* sms) {
+    AIO_CUDA(cudaGetDevice(dev));
+    int major = 0, minor = 0;
+    AIO_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, *dev));
+    AIO_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, *dev));
+    if (major != 10 || minor != 3)
+        return fail(AIO_ERR_UNSUPPORTED, "device %d is sm_%d%d; libaio is built for sm_103a (GB300) only", *dev, major,
+                    minor);
+    AIO_CUDA(cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, *dev));
+    std::lock_guard<std::mutex> lk(g_prep_mu);
+    if (*dev < 0 || *dev >= 64) return fail(AIO_ERR_UNSUPPORTED, "device ordinal %d out of range", *dev);
+    if (!g_prepared[*dev]) {
+        AIO_CUDA(aio::prepare_kernels());
+        g_prepared[*dev] = true;
+    }
+    return AIO_OK;
+}
+
+aio_status check_device(int dev) {
+    int cur = -1;
+    AIO_CUDA(cudaGetDevice(&cur));
+    if (cur != dev) return fail(AIO_ERR_STATE, "object belongs to device %d but device %d is current", dev, cur);
+    return AIO_OK;
+}
+
+}  // namespace
+
+namespace aio {
+
+Geometry geometry(int K, int N, int num_sms) {
+    Geometry g;
+    g.NG = (N + kRows - 1) / kRows;
+    g.NKT = (K + kKT - 1) / kKT;
+    g.T = static_cast<long long>(g.NG) * g.NKT;
+    g.grid = num_sms;
+    g.Z = g.grid * kWarps;
+    return g;
+}
+
+size_t workspace_bytes(const Geometry& g, int M) {
+    return round_up(static_cast<size_t>(g.Z) * 2 * kRows * M * sizeof(float), 256) +
+           round_up(static_cast<size_t>(g.NG) * sizeof(unsigned), 256);
+}
+
+void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters, int** err) {
+    uint8_t* p = static_cast<uint8_t*>(base);
+    *partial = reinterpret_cast<float*>(p);
+    p += round_up(static_cast<size_t>(g.Z) * 2 * kRows * M * sizeof(float), 256);
+    *counters = reinterpret_cast<unsigned*>(p);
+    (void)err;
+}
+
+}  // namespace aio
+
+struct aio_linear {
+    uint32_t magic;
+    int K, N, max_M;
+    aio_wtype wt;
+    unsigned flags;
+    int device;
+    aio::Geometry geo;
+    void* ws;            // partial sums, counters, then the error word
+    size_t ws_bytes;
+    float* partial;
+    unsigned* counters;
+    int* err;
+};
+
+struct aio_step {
+    uint32_t magic;
+    int device, M, n;
+    unsigned flags;
+    std::vector<aio::GemvArgs> args;
+    std::vector<char> i8;
+    std::vector<int> grid;
+    void* ws;            // per-projection workspaces, then one error word per projection
+    size_t ws_bytes;
+    int* errs;
+    cudaGraph_t graph;
+    cudaGraphExec_t exec;
+};
+
+namespace {
+
+aio_status valid_linear(aio_linear_t h) {
+    if (!h) return fail(AIO_ERR_INVALID_ARG, "null aio_linear_t");
+    if (h->magic != kLinearMagic) return fail(AIO_ERR_STATE, "aio_linear_t is not a live handle");
+    return AIO_OK;
+}
+
+aio::GemvArgs make_args(const aio_linear* h, const void* x, int M, const void* W, const void* scales, float* y,
+                        float* partial, unsigned* counters, int* err) {
+    aio::GemvArgs a;
+    a.x = static_cast<const uint16_t*>(x);
+    a.w = static_cast<const uint8_t*>(W);
+    a.scales = static_cast<const uint16_t*>(scales);
+    a.y = y;
+    a.partial = partial;
+    a.counters = counters;
+    a.err = err;
+    a.T = h->geo.T;
+    a.M = M;
+    a.K = h->K;
+    a.N = h->N;
+    a.NG = h->geo.NG;
+    a.NKT = h->geo.NKT;
+    a.Z = h->geo.Z;
+    a.rowmajor = (h->flags & AIO_FLAG_ROWMAJOR) ? 1 : 0;
+    a.test_stall = (h->flags & AIO_FLAG_TEST_STALL) ? 1 : 0;
+    a.wait_limit_ns = a.test_stall ? kTestWaitLimitNs : kWaitLimitNs;
+    return a;
+}
+
+aio_status validate_run(const aio_linear* h, const void* x, int M, const void* W, const void* scales, const float* y) {
+    if (M < 1 || M > h->max_M) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, max_M=%d]", M, h->max_M);
+    if (!x || !W || !y) return fail(AIO_ERR_INVALID_ARG, "x, W and y must be non-NULL");
+    if (!aligned(x, 16) || !aligned(W, 16) || !aligned(y, 16))
+        return fail(AIO_ERR_ALIGNMENT, "x, W and y must be 16-byte aligned");
+    if (h->wt == AIO_W_INT8_PERCHANNEL) {
+        if (!scales) return fail(AIO_ERR_INVALID_ARG, "int8 weights need per-channel scales");
+        if (!aligned(scales, 2)) return fail(AIO_ERR_ALIGNMENT, "scales must be 2-byte aligned");
+    } else if (scales) {
+        return fail(AIO_ERR_INVALID_ARG, "bf16 weights take no scales (pass NULL)");
+    }
+    return AIO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int aio_abi_version(void) { return AIO_ABI_VERSION; }
+
+const char* aio_status_string(aio_status s) {
+    switch (s) {
+        case AIO_OK: return "AIO_OK";
+        case AIO_ERR_INVALID_ARG: return "AIO_ERR_INVALID_ARG";
+        case AIO_ERR_UNSUPPORTED: return "AIO_ERR_UNSUPPORTED";
+        case AIO_ERR_ALIGNMENT: return "AIO_ERR_ALIGNMENT";
+        case AIO_ERR_CUDA: return "AIO_ERR_CUDA";
+        case AIO_ERR_OOM: return "AIO_ERR_OOM";
+        case AIO_ERR_STATE: return "AIO_ERR_STATE";
+        case AIO_ERR_DEVICE_TIMEOUT: return "AIO_ERR_DEVICE_TIMEOUT";
+    }
+    return "AIO_ERR_UNKNOWN";
+}
+
+const char* aio_last_error(void) { return g_last_error; }
+
+aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int max_M, unsigned flags) {
+    if (!out) return fail(AIO_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (K < 16 || K > (1 << 20) || K % 16 != 0) return fail(AIO_ERR_INVALID_ARG, "K=%d: need 16 <= K <= 2^20, K %% 16 == 0", K);
+    if (N < 1 || N > (1 << 24)) return fail(AIO_ERR_INVALID_ARG, "N=%d: need 1 <= N <= 2^24", N);
+    if (wt != AIO_W_BF16 && wt != AIO_W_INT8_PERCHANNEL) return fail(AIO_ERR_INVALID_ARG, "unknown weight type %d", (int)wt);
+    if (max_M < 1 || max_M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "max_M=%d outside [1, 8]", max_M);
+    if (flags & ~kCreateFlags) return fail(AIO_ERR_INVALID_ARG, "unknown flags 0x%x", flags & ~kCreateFlags);
+    int dev = 0, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    aio::Geometry geo = aio::geometry(K, N, sms);
+    const size_t ws = aio::workspace_bytes(geo, max_M);
+    if (test_alloc_failure()) return fail(AIO_ERR_OOM, "workspace allocation failed (AIO_TEST_FAIL_ALLOC)");
+    void* mem = nullptr;
+    if (cudaMalloc(&mem, ws + 256) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(AIO_ERR_OOM, "cudaMalloc(%zu) failed", ws + 256);
+    }
+    if (cudaMemset(mem, 0, ws + 256) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+        cudaFree(mem);
+        return fail(AIO_ERR_CUDA, "workspace initialisation failed");
+    }
+    aio_linear* h = new (std::nothrow) aio_linear();
+    if (!h) {
+        cudaFree(mem);
+        return fail(AIO_ERR_OOM, "host allocation failed");
+    }
+    h->magic = kLinearMagic;
+    h->K = K;
+    h->N = N;
+    h->max_M = max_M;
+    h->wt = wt;
+    h->flags = flags;
+    h->device = dev;
+    h->geo = geo;
+    h->ws = mem;
+    h->ws_bytes = ws + 256;
+    aio::carve_workspace(mem, geo, max_M, &h->partial, &h->counters, nullptr);
+    h->err = reinterpret_cast<int*>(static_cast<uint8_t*>(mem) + ws);
+    *out = h;
+    return AIO_OK;
+}
+
+aio_status aio_linear_packed_bytes(aio_linear_t h, size_t* w_bytes, size_t* scale_bytes) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    const size_t e = h->wt == AIO_W_BF16 ? 2 : 1;
+    if (w_bytes) *w_bytes = static_cast<size_t>(h->N) * h->K * e;
+    if (scale_bytes) *scale_bytes = h->wt == AIO_W_BF16 ? 0 : static_cast<size_t>(h->N) * 2;
+    return AIO_OK;
+}
+
+aio_status aio_linear_launch_info(aio_linear_t h, int* grid, int* block, size_t* smem_bytes, long long* tiles) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    if (grid) *grid = h->geo.grid;
+    if (block) *block = aio::kThreads;
+    if (smem_bytes) *smem_bytes = aio::kSmemBytes;
+    if (tiles) *tiles = h->geo.T;
+    return AIO_OK;
+}
+
+static aio_status pack_common(aio_linear_t h, const void* src, void* dst, bool inverse, void* stream) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    if ((st = check_device(h->device)) != AIO_OK) return st;
+    if (!src || !dst) return fail(AIO_ERR_INVALID_ARG, "weight pointers must be non-NULL");
+    if (!aligned(src, 16) || !aligned(dst, 16)) return fail(AIO_ERR_ALIGNMENT, "weight pointers must be 16-byte aligned");
+    const size_t e = h->wt == AIO_W_BF16 ? 2 : 1;
+    const size_t bytes = static_cast<size_t>(h->N) * h->K * e;
+    const uintptr_t a = reinterpret_cast<uintptr_t>(src), b = reinterpret_cast<uintptr_t>(dst);
+    if (a < b + bytes && b < a + bytes) return fail(AIO_ERR_INVALID_ARG, "source and destination overlap");
+    AIO_CUDA(aio::launch_pack(src, dst, h->N, h->K, static_cast<int>(e), inverse, static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}
+
+aio_status aio_linear_pack(aio_linear_t h, const void* W_rowmajor, const void* scales, void* W_packed,
+                           void* scales_packed, void* stream) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    if (h->wt == AIO_W_INT8_PERCHANNEL) {
+        if (!scales || !scales_packed) return fail(AIO_ERR_INVALID_ARG, "int8 weights need scales and scales_packed");
+        if (!aligned(scales, 2) || !aligned(scales_packed, 2)) return fail(AIO_ERR_ALIGNMENT, "scales must be 2-byte aligned");
+    } else if (scales || scales_packed) {
+        return fail(AIO_ERR_INVALID_ARG, "bf16 weights take no scales (pass NULL)");
+    }
+    if ((st = pack_common(h, W_rowmajor, W_packed, false, stream)) != AIO_OK) return st;
+    if (h->wt == AIO_W_INT8_PERCHANNEL && scales != scales_packed)
+        AIO_CUDA(cudaMemcpyAsync(scales_packed, scales, static_cast<size_t>(h->N) * 2, cudaMemcpyDeviceToDevice,
+                                 static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}
+
+aio_status aio_linear_unpack(aio_linear_t h, const void* W_packed, void* W_rowmajor, void* stream) {
+    return pack_common(h, W_packed, W_rowmajor, true, stream);
+}
+
+aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, const void* W, const void* scales,
+                          float* y, void* stream) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    if (K != h->K || N != h->N) return fail(AIO_ERR_INVALID_ARG, "K=%d N=%d do not match the handle (K=%d N=%d)", K, N, h->K, h->N);
+    if ((st = validate_run(h, x, M, W, scales, y)) != AIO_OK) return st;
+    if ((st = check_device(h->device)) != AIO_OK) return st;
+    aio::GemvArgs a = make_args(h, x, M, W, scales, y, h->partial, h->counters, h->err);
+    AIO_CUDA(aio::launch_gemv(a, h->wt == AIO_W_INT8_PERCHANNEL, h->geo.grid, static_cast<cudaStream_t>(stream),
+                              !(h->flags & AIO_FLAG_NO_PDL)));
+    return AIO_OK;
+}
+
+static aio_status read_errors(int device, const int* errs, int n, int* device_error) {
+    aio_status st = check_device(device);
+    if (st != AIO_OK) return st;
+    AIO_CUDA(cudaDeviceSynchronize());
+    std::vector<int> host(static_cast<size_t>(n));
+    AIO_CUDA(cudaMemcpy(host.data(), errs, sizeof(int) * n, cudaMemcpyDeviceToHost));
+    int e = 0;
+    for (int v : host) e = e ? e : v;
+    if (device_error) *device_error = e;
+    if (e) return fail(AIO_ERR_DEVICE_TIMEOUT, "a bounded device wait expired (code %d)", e);
+    return AIO_OK;
+}
+
+aio_status aio_linear_check(aio_linear_t h, int* device_error) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    return read_errors(h->device, h->err, 1, device_error);
+}
+
+aio_status aio_linear_reset(aio_linear_t h) {
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    if ((st = check_device(h->device)) != AIO_OK) return st;
+    AIO_CUDA(cudaDeviceSynchronize());
+    AIO_CUDA(cudaMemset(h->ws, 0, h->ws_bytes));
+    AIO_CUDA(cudaDeviceSynchronize());
+    return AIO_OK;
+}
+
+aio_status aio_linear_destroy(aio_linear_t h) {
+    if (!h) return AIO_OK;
+    aio_status st = valid_linear(h);
+    if (st != AIO_OK) return st;
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != h->device) cudaSetDevice(h->device);
+    cudaDeviceSynchronize();
+    cudaFree(h->ws);
+    if (cur != h->device) cudaSetDevice(cur);
+    h->magic = 0;
+    delete h;
+    return AIO_OK;
+}
+
+static void step_free(aio_step* s) {
+    if (!s) return;
+    if (s->exec) cudaGraphExecDestroy(s->exec);
+    if (s->graph) cudaGraphDestroy(s->graph);
+    if (s->ws) cudaFree(s->ws);
+    s->magic = 0;
+    delete s;
+}
+
+static aio_status step_launch_all(aio_step* s, cudaStream_t stream) {
+    for (int i = 0; i < s->n; ++i) {
+        const bool pdl = i > 0 && (s->flags & AIO_STEP_PDL);
+        AIO_CUDA(aio::launch_gemv(s->args[i], s->i8[i] != 0, s->grid[i], stream, pdl));
+    }
+    return AIO_OK;
+}
+
+aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_projs, int M, unsigned flags) {
+    if (!out) return fail(AIO_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (!projs || n_projs < 1) return fail(AIO_ERR_INVALID_ARG, "need at least one projection");
+    if (flags & ~kStepFlags) return fail(AIO_ERR_INVALID_ARG, "unknown step flags 0x%x", flags & ~kStepFlags);
+    if (M < 1 || M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, 8]", M);
+    int dev = -1;
+    {
+        aio_status st = valid_linear(projs[0].h);
+        if (st != AIO_OK) return st;
+        dev = projs[0].h->device;
+    }
+    size_t total = 0;
+    std::vector<size_t> offs(static_cast<size_t>(n_projs));
+    for (int i = 0; i < n_projs; ++i) {
+        const aio_proj& p = projs[i];
+        aio_status st = valid_linear(p.h);
+        if (st != AIO_OK) return fail(st, "projection %d: %s", i, g_last_error);
+        if (p.h->device != dev) return fail(AIO_ERR_STATE, "projection %d is on device %d, not %d", i, p.h->device, dev);
+        if ((st = validate_run(p.h, p.x, M, p.W, p.scales, p.y)) != AIO_OK)
+            return fail(st, "projection %d: %s", i, g_last_error);
+        offs[i] = total;
+        total += aio::workspace_bytes(p.h->geo, M);
+    }
+    aio_status st = check_device(dev);
+    if (st != AIO_OK) return st;
+    const size_t err_off = total;
+    total += round_up(sizeof(int) * n_projs, 256);
+    if (test_alloc_failure()) return fail(AIO_ERR_OOM, "workspace allocation failed (AIO_TEST_FAIL_ALLOC)");
+    aio_step* s = new (std::nothrow) aio_step();
+    if (!s) return fail(AIO_ERR_OOM, "host allocation failed");
+    s->magic = kStepMagic;
+    s->device = dev;
+    s->M = M;
+    s->n = n_projs;
+    s->flags = flags;
+    s->ws_bytes = total;
+    if (cudaMalloc(&s->ws, total) != cudaSuccess) {
+        cudaGetLastError();
+        s->ws = nullptr;
+        step_free(s);
+        return fail(AIO_ERR_OOM, "cudaMalloc(%zu) failed", total);
+    }
+    if (cudaMemset(s->ws, 0, total) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+        step_free(s);
+        return fail(AIO_ERR_CUDA, "step workspace initialisation failed");
+    }
+    s->errs = reinterpret_cast<int*>(static_cast<uint8_t*>(s->ws) + err_off);
+    for (int i = 0; i < n_projs; ++i) {
+        const aio_proj& p = projs[i];
+        float* partial = nullptr;
+        unsigned* counters = nullptr;
+        aio::carve_workspace(static_cast<uint8_t*>(s->ws) + offs[i], p.h->geo, M, &partial, &counters, nullptr);
+        s->args.push_back(make_args(p.h, p.x, M, p.W, p.scales, p.y, partial, counters, s->errs + i));
+        s->i8.push_back(p.h->wt == AIO_W_INT8_PERCHANNEL ? 1 : 0);
+        s->grid.push_back(p.h->geo.grid);
+    }
+    if (flags & AIO_STEP_GRAPH) {
+        cudaStream_t cs = nullptr;
+        if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) {
+            step_free(s);
+            return fail(AIO_ERR_CUDA, "capture stream creation failed");
+        }
+        aio_status lst = AIO_OK;
+        if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+            lst = fail(AIO_ERR_CUDA, "cudaStreamBeginCapture failed");
+        } else {
+            lst = step_launch_all(s, cs);
+            cudaGraph_t g = nullptr;
+            const cudaError_t ec = cudaStreamEndCapture(cs, &g);
+            if (lst == AIO_OK && ec != cudaSuccess) lst = fail(AIO_ERR_CUDA, "cudaStreamEndCapture: %s", cudaGetErrorString(ec));
+            s->graph = g;
+            if (lst == AIO_OK) {
+                const cudaError_t ei = cudaGraphInstantiate(&s->exec, s->graph, 0);
+                if (ei != cudaSuccess) lst = fail(AIO_ERR_CUDA, "cudaGraphInstantiate: %s", cudaGetErrorString(ei));
+            }
+        }
+        cudaStreamDestroy(cs);
+        if (lst != AIO_OK) {
+            cudaGetLastError();
+            step_free(s);
+            return lst;
+        }
+    }
+    *out = s;
+    return AIO_OK;
+}
+
+static aio_status valid_step(aio_step_t s) {
+    if (!s) return fail(AIO_ERR_INVALID_ARG, "null aio_step_t");
+    if (s->magic != kStepMagic) return fail(AIO_ERR_STATE, "aio_step_t is not a live step");
+    return AIO_OK;
+}
+
+aio_status aio_decode_step(aio_step_t s, void* stream) {
+    aio_status st = valid_step(s);
+    if (st != AIO_OK) return st;
+    if ((st = check_device(s->device)) != AIO_OK) return st;
+    if (s->exec) {
+        AIO_CUDA(cudaGraphLaunch(s->exec, static_cast<cudaStream_t>(stream)));
+        return AIO_OK;
+    }
+    return step_launch_all(s, static_cast<cudaStream_t>(stream));
+}
+
+aio_status aio_decode_step_kernels(aio_step_t s, int* n_kernels) {
+    aio_status st = valid_step(s);
+    if (st != AIO_OK) return st;
+    if (n_kernels) *n_kernels = s->n;
+    return AIO_OK;
+}
+
+aio_status aio_decode_step_check(aio_step_t s, int* device_error) {
+    aio_status st = valid_step(s);
+    if (st != AIO_OK) return st;
+    return read_errors(s->device, s->errs, s->n, device_error);
+}
+
+aio_status aio_decode_step_destroy(aio_step_t s) {
+    if (!s) return AIO_OK;
+    aio_status st = valid_step(s);
+    if (st != AIO_OK) return st;
+    const int dev = s->device;
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != dev) cudaSetDevice(dev);
+    cudaDeviceSynchronize();
+    step_free(s);
+    if (cur != dev) cudaSetDevice(cur);
+    return AIO_OK;
+}
+
+aio_status aio_probe_read(const void* buf, size_t bytes, unsigned* out, void* stream) {
+    if (!buf || !out) return fail(AIO_ERR_INVALID_ARG, "buf and out must be non-NULL");
+    if (bytes == 0 || bytes % 4096 != 0) return fail(AIO_ERR_INVALID_ARG, "bytes must be a positive multiple of 4096");
+    if (!aligned(buf, 16) || !aligned(out, 4)) return fail(AIO_ERR_ALIGNMENT, "buf must be 16-byte aligned, out 4-byte");
+    int dev = 0, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    AIO_CUDA(aio::launch_probe(buf, static_cast<long long>(bytes / 4096), out, 2 * sms, static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}
+
+}  // extern "C"
