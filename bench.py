@@ -3,8 +3,8 @@
 equivalent decode tokens/s on GB300.
 
 A step is one pass of every projection of a decoder (Sec. 3.1: each generated token streams all
-weights from HBM): 4 projections per layer plus the lm_head, replayed as one CUDA graph with
-programmatic dependent launch.  Default workload: the 7B-class decode step at M=1 in bf16
+weights from HBM): 4 projections per layer plus the lm_head, streamed by one persistent
+cooperative kernel launch (one CUDA graph node).  Default workload: the 7B-class decode step at M=1 in bf16
 (32 layers, 129 projections, 13.21 GB of weights per token), synthetic seeded weights.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
@@ -230,7 +230,8 @@ def run_ours(args, wl):
     setup_s = time.perf_counter() - t_setup
     stream = torch.cuda.Stream()
     sh = stream.cuda_stream
-    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL
+    flags = {"persistent": aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT,
+             "chain": aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL}[args.step_mode]
     step = dw.step_handle(M, flags)
     n_kernels = aio.aio_decode_step_kernels(step)
     wbytes = dw.weight_bytes()
@@ -358,7 +359,7 @@ def run_ours(args, wl):
                 "weight_bytes_per_token": wbytes,
                 "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                 "l2": "inputs larger than L2 (every step streams all weights, >= 2.39 GB)",
-                "graph": "one CUDA graph per step, PDL between projections",
+                "step_mode": args.step_mode,
             },
             "tokens_per_s": round(tokens, 2),
             "verified_tokens_per_s_upper_bound": round(tokens * M, 2),
@@ -366,7 +367,7 @@ def run_ours(args, wl):
             "pct_of_nominal_8tbs": round(100 * gbs_rank / NOMINAL_HBM_GBS, 2),
             "roofline": {
                 "bound": "hbm",
-                "kernel": f"aio_gemv_kernel<M={M}, {'int8' if dw.i8 else 'bf16'}>",
+                "kernel": f"aio_stream_kernel<M={M}, {'int8' if dw.i8 else 'bf16'}>",
                 "achieved": round(gbs_rank, 2),
                 "peak": peak,
                 "unit": "GB/s",
@@ -406,6 +407,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-frac", type=float, default=0.125)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--step-mode", choices=["persistent", "chain"], default="persistent",
+                    help="one cooperative launch per step (default) or one launch per projection")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")

@@ -70,8 +70,13 @@ typedef enum {
                                       AIO_ERR_DEVICE_TIMEOUT; outputs are then undefined */
 
 /* aio_decode_step_create flags */
-#define AIO_STEP_GRAPH 0x1u        /* capture the whole step into one CUDA graph (one launch per step) */
-#define AIO_STEP_PDL   0x2u        /* programmatic dependent launch between consecutive projections */
+#define AIO_STEP_GRAPH      0x1u   /* capture the step's launches into one CUDA graph (one launch per step) */
+#define AIO_STEP_PDL        0x2u   /* chain mode: programmatic dependent launch between projections */
+#define AIO_STEP_PERSISTENT 0x4u   /* one cooperative launch streams every projection: each SM keeps a deep
+                                      ring of weight tiles in flight across projection boundaries, and a
+                                      bounded grid-wide counter orders projection i+1's x reads after
+                                      projection i.  Needs one weight type for all projections.  Without
+                                      this flag the step is a chain of one launch per projection. */
 
 /* Packed weight layout written by aio_linear_pack (a permutation of W, no padding):
  * rows are grouped 8 at a time and each group is cut into tiles of 256 k-columns;
@@ -165,16 +170,20 @@ aio_status aio_linear_destroy(aio_linear_t h);
  * reading its x only after projection i has completed (Sec. 3.1: every weight of every layer is
  * streamed once per token).  Pointer values are captured at creation: later calls rewrite the
  * buffers' contents, never their addresses.  1 <= M <= every handle's max_M.  The step owns a
- * private workspace per projection (so consecutive projections may overlap under PDL).
- * flags: AIO_STEP_GRAPH and/or AIO_STEP_PDL.  Errors: INVALID_ARG, ALIGNMENT, STATE, OOM, CUDA.
+ * private workspace per projection (so consecutive projections may overlap), a device copy of
+ * the projection list, and per-projection completion counters; runs of one step must not overlap
+ * in time.  flags: AIO_STEP_* bits.  Errors: INVALID_ARG, ALIGNMENT, STATE, UNSUPPORTED, OOM, CUDA.
  */
 aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_projs, int M, unsigned flags);
 
 /* Enqueue one decode step on stream (one graph launch with AIO_STEP_GRAPH). */
 aio_status aio_decode_step(aio_step_t step, void* stream);
 
-/* Number of kernels one aio_decode_step launches. */
+/* Number of kernels one aio_decode_step launches (1 in persistent mode, else one per projection). */
 aio_status aio_decode_step_kernels(aio_step_t step, int* n_kernels);
+
+/* Clear the step's workspace counters and error words (needed only after a device error). */
+aio_status aio_decode_step_reset(aio_step_t step);
 
 /* Synchronise the device, then report the step's device error word (see aio_linear_check). */
 aio_status aio_decode_step_check(aio_step_t step, int* device_error);

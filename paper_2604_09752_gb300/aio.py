@@ -38,6 +38,7 @@ AIO_FLAG_NO_PDL = 0x2
 AIO_FLAG_TEST_STALL = 0x100
 AIO_STEP_GRAPH = 0x1
 AIO_STEP_PDL = 0x2
+AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 8
 AIO_K_TILE = 256
 for _name, _val in re.findall(r"#define\s+(AIO_\w+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", _hdr):
@@ -78,6 +79,7 @@ _SIGS = {
     "aio_decode_step": (_int, [_vp, _vp]),
     "aio_decode_step_kernels": (_int, [_vp, ctypes.POINTER(_int)]),
     "aio_decode_step_check": (_int, [_vp, ctypes.POINTER(_int)]),
+    "aio_decode_step_reset": (_int, [_vp]),
     "aio_decode_step_destroy": (_int, [_vp]),
     "aio_probe_read": (_int, [_vp, _sz, _vp, _vp]),
 }
@@ -153,7 +155,7 @@ def aio_linear_destroy(h: int):
     _check(_lib.aio_linear_destroy(h), "aio_linear_destroy")
 
 
-def aio_decode_step_create(projs, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP_PDL) -> int:
+def aio_decode_step_create(projs, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP_PERSISTENT) -> int:
     """projs: sequence of (h, x, W, scales, y) integer addresses (scales may be None)."""
     arr = (aio_proj * len(projs))(*[aio_proj(*p) for p in projs])
     s = _vp()
@@ -175,6 +177,10 @@ def aio_decode_step_check(step: int) -> int:
     e = _int()
     _check(_lib.aio_decode_step_check(step, ctypes.byref(e)), "aio_decode_step_check")
     return e.value
+
+
+def aio_decode_step_reset(step: int):
+    _check(_lib.aio_decode_step_reset(step), "aio_decode_step_reset")
 
 
 def aio_decode_step_destroy(step: int):

@@ -19,7 +19,7 @@ namespace {
 constexpr uint32_t kLinearMagic = 0xA10113EAu;
 constexpr uint32_t kStepMagic = 0xA1057E90u;
 constexpr unsigned kCreateFlags = AIO_FLAG_ROWMAJOR | AIO_FLAG_NO_PDL | AIO_FLAG_TEST_STALL;
-constexpr unsigned kStepFlags = AIO_STEP_GRAPH | AIO_STEP_PDL;
+constexpr unsigned kStepFlags = AIO_STEP_GRAPH | AIO_STEP_PDL | AIO_STEP_PERSISTENT;
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;      // 1 s: a healthy wait takes microseconds
 constexpr unsigned long long kTestWaitLimitNs = 20000000ull;    // 20 ms for AIO_FLAG_TEST_STALL
 
@@ -96,12 +96,11 @@ size_t workspace_bytes(const Geometry& g, int M) {
            round_up(static_cast<size_t>(g.NG) * sizeof(unsigned), 256);
 }
 
-void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters, int** err) {
+void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters) {
     uint8_t* p = static_cast<uint8_t*>(base);
     *partial = reinterpret_cast<float*>(p);
     p += round_up(static_cast<size_t>(g.Z) * 2 * kRows * M * sizeof(float), 256);
     *counters = reinterpret_cast<unsigned*>(p);
-    (void)err;
 }
 
 }  // namespace aio
@@ -124,10 +123,13 @@ struct aio_step {
     uint32_t magic;
     int device, M, n;
     unsigned flags;
-    std::vector<aio::GemvArgs> args;
-    std::vector<char> i8;
-    std::vector<int> grid;
-    void* ws;            // per-projection workspaces, then one error word per projection
+    bool persistent;
+    bool i8;                             // weight type of every projection (persistent mode)
+    int grid;
+    std::vector<aio::StreamArgs> chain;  // per-projection launches (chain mode)
+    std::vector<char> chain_i8;
+    aio::StreamArgs whole;               // one launch over the device descriptor array (persistent mode)
+    void* ws;                            // workspaces, descriptors, done counters, error words
     size_t ws_bytes;
     int* errs;
     cudaGraph_t graph;
@@ -142,24 +144,35 @@ aio_status valid_linear(aio_linear_t h) {
     return AIO_OK;
 }
 
-aio::GemvArgs make_args(const aio_linear* h, const void* x, int M, const void* W, const void* scales, float* y,
-                        float* partial, unsigned* counters, int* err) {
-    aio::GemvArgs a;
-    a.x = static_cast<const uint16_t*>(x);
-    a.w = static_cast<const uint8_t*>(W);
-    a.scales = static_cast<const uint16_t*>(scales);
-    a.y = y;
-    a.partial = partial;
-    a.counters = counters;
+aio::ProjDesc make_desc(const aio_linear* h, const void* x, const void* W, const void* scales, float* y,
+                        float* partial, unsigned* counters) {
+    aio::ProjDesc d = {};
+    d.x = static_cast<const uint16_t*>(x);
+    d.w = static_cast<const uint8_t*>(W);
+    d.scales = static_cast<const uint16_t*>(scales);
+    d.y = y;
+    d.partial = partial;
+    d.counters = counters;
+    d.T = h->geo.T;
+    d.K = h->K;
+    d.N = h->N;
+    d.NG = h->geo.NG;
+    d.NKT = h->geo.NKT;
+    d.rowmajor = (h->flags & AIO_FLAG_ROWMAJOR) ? 1 : 0;
+    d.uniform = (!d.rowmajor && h->N % aio::kRows == 0 && h->K % aio::kKT == 0) ? 1 : 0;
+    return d;
+}
+
+aio::StreamArgs single_args(const aio_linear* h, const aio::ProjDesc& d, int M, int* err) {
+    aio::StreamArgs a = {};
+    a.projs = nullptr;
+    a.one = d;
+    a.done = nullptr;
+    a.exit_count = nullptr;
     a.err = err;
-    a.T = h->geo.T;
+    a.nproj = 1;
     a.M = M;
-    a.K = h->K;
-    a.N = h->N;
-    a.NG = h->geo.NG;
-    a.NKT = h->geo.NKT;
     a.Z = h->geo.Z;
-    a.rowmajor = (h->flags & AIO_FLAG_ROWMAJOR) ? 1 : 0;
     a.test_stall = (h->flags & AIO_FLAG_TEST_STALL) ? 1 : 0;
     a.wait_limit_ns = a.test_stall ? kTestWaitLimitNs : kWaitLimitNs;
     return a;
@@ -239,7 +252,7 @@ aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int 
     h->geo = geo;
     h->ws = mem;
     h->ws_bytes = ws + 256;
-    aio::carve_workspace(mem, geo, max_M, &h->partial, &h->counters, nullptr);
+    aio::carve_workspace(mem, geo, max_M, &h->partial, &h->counters);
     h->err = reinterpret_cast<int*>(static_cast<uint8_t*>(mem) + ws);
     *out = h;
     return AIO_OK;
@@ -306,9 +319,9 @@ aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, co
     if (K != h->K || N != h->N) return fail(AIO_ERR_INVALID_ARG, "K=%d N=%d do not match the handle (K=%d N=%d)", K, N, h->K, h->N);
     if ((st = validate_run(h, x, M, W, scales, y)) != AIO_OK) return st;
     if ((st = check_device(h->device)) != AIO_OK) return st;
-    aio::GemvArgs a = make_args(h, x, M, W, scales, y, h->partial, h->counters, h->err);
-    AIO_CUDA(aio::launch_gemv(a, h->wt == AIO_W_INT8_PERCHANNEL, h->geo.grid, static_cast<cudaStream_t>(stream),
-                              !(h->flags & AIO_FLAG_NO_PDL)));
+    const aio::StreamArgs a = single_args(h, make_desc(h, x, W, scales, y, h->partial, h->counters), M, h->err);
+    AIO_CUDA(aio::launch_stream(a, h->wt == AIO_W_INT8_PERCHANNEL, h->geo.grid, static_cast<cudaStream_t>(stream),
+                                !(h->flags & AIO_FLAG_NO_PDL), false));
     return AIO_OK;
 }
 
@@ -366,9 +379,13 @@ static void step_free(aio_step* s) {
 }
 
 static aio_status step_launch_all(aio_step* s, cudaStream_t stream) {
+    if (s->persistent) {
+        AIO_CUDA(aio::launch_stream(s->whole, s->i8, s->grid, stream, false, true));
+        return AIO_OK;
+    }
     for (int i = 0; i < s->n; ++i) {
         const bool pdl = i > 0 && (s->flags & AIO_STEP_PDL);
-        AIO_CUDA(aio::launch_gemv(s->args[i], s->i8[i] != 0, s->grid[i], stream, pdl));
+        AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false));
     }
     return AIO_OK;
 }
@@ -379,12 +396,14 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     if (!projs || n_projs < 1) return fail(AIO_ERR_INVALID_ARG, "need at least one projection");
     if (flags & ~kStepFlags) return fail(AIO_ERR_INVALID_ARG, "unknown step flags 0x%x", flags & ~kStepFlags);
     if (M < 1 || M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, 8]", M);
+    const bool persistent = (flags & AIO_STEP_PERSISTENT) != 0;
     int dev = -1;
     {
         aio_status st = valid_linear(projs[0].h);
         if (st != AIO_OK) return st;
         dev = projs[0].h->device;
     }
+    const aio_wtype wt0 = projs[0].h->wt;
     size_t total = 0;
     std::vector<size_t> offs(static_cast<size_t>(n_projs));
     for (int i = 0; i < n_projs; ++i) {
@@ -392,6 +411,8 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
         aio_status st = valid_linear(p.h);
         if (st != AIO_OK) return fail(st, "projection %d: %s", i, g_last_error);
         if (p.h->device != dev) return fail(AIO_ERR_STATE, "projection %d is on device %d, not %d", i, p.h->device, dev);
+        if (persistent && p.h->wt != wt0)
+            return fail(AIO_ERR_UNSUPPORTED, "a persistent step needs one weight type (projection %d differs)", i);
         if ((st = validate_run(p.h, p.x, M, p.W, p.scales, p.y)) != AIO_OK)
             return fail(st, "projection %d: %s", i, g_last_error);
         offs[i] = total;
@@ -399,6 +420,16 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     }
     aio_status st = check_device(dev);
     if (st != AIO_OK) return st;
+    const int grid = projs[0].h->geo.grid;
+    if (persistent) {
+        int blocks = 0;
+        AIO_CUDA(aio::occupancy(wt0 == AIO_W_INT8_PERCHANNEL, M, &blocks));
+        if (blocks < 1) return fail(AIO_ERR_UNSUPPORTED, "the stream kernel cannot be resident on an SM");
+    }
+    const size_t desc_off = total;
+    total += round_up(sizeof(aio::ProjDesc) * n_projs, 256);
+    const size_t done_off = total;
+    total += round_up(sizeof(unsigned) * (n_projs + 1), 256);
     const size_t err_off = total;
     total += round_up(sizeof(int) * n_projs, 256);
     if (test_alloc_failure()) return fail(AIO_ERR_OOM, "workspace allocation failed (AIO_TEST_FAIL_ALLOC)");
@@ -409,6 +440,9 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     s->M = M;
     s->n = n_projs;
     s->flags = flags;
+    s->persistent = persistent;
+    s->i8 = wt0 == AIO_W_INT8_PERCHANNEL;
+    s->grid = grid;
     s->ws_bytes = total;
     if (cudaMalloc(&s->ws, total) != cudaSuccess) {
         cudaGetLastError();
@@ -416,19 +450,34 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
         step_free(s);
         return fail(AIO_ERR_OOM, "cudaMalloc(%zu) failed", total);
     }
-    if (cudaMemset(s->ws, 0, total) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
-        step_free(s);
-        return fail(AIO_ERR_CUDA, "step workspace initialisation failed");
-    }
-    s->errs = reinterpret_cast<int*>(static_cast<uint8_t*>(s->ws) + err_off);
+    uint8_t* base = static_cast<uint8_t*>(s->ws);
+    s->errs = reinterpret_cast<int*>(base + err_off);
+    std::vector<aio::ProjDesc> descs;
     for (int i = 0; i < n_projs; ++i) {
         const aio_proj& p = projs[i];
         float* partial = nullptr;
         unsigned* counters = nullptr;
-        aio::carve_workspace(static_cast<uint8_t*>(s->ws) + offs[i], p.h->geo, M, &partial, &counters, nullptr);
-        s->args.push_back(make_args(p.h, p.x, M, p.W, p.scales, p.y, partial, counters, s->errs + i));
-        s->i8.push_back(p.h->wt == AIO_W_INT8_PERCHANNEL ? 1 : 0);
-        s->grid.push_back(p.h->geo.grid);
+        aio::carve_workspace(base + offs[i], p.h->geo, M, &partial, &counters);
+        descs.push_back(make_desc(p.h, p.x, p.W, p.scales, p.y, partial, counters));
+        s->chain.push_back(single_args(p.h, descs.back(), M, s->errs + i));
+        s->chain_i8.push_back(p.h->wt == AIO_W_INT8_PERCHANNEL ? 1 : 0);
+    }
+    aio::StreamArgs w = {};
+    w.projs = reinterpret_cast<const aio::ProjDesc*>(base + desc_off);
+    w.done = reinterpret_cast<unsigned*>(base + done_off);
+    w.exit_count = w.done + n_projs;
+    w.err = s->errs;
+    w.nproj = n_projs;
+    w.M = M;
+    w.Z = projs[0].h->geo.Z;
+    w.test_stall = 0;
+    w.wait_limit_ns = kWaitLimitNs;
+    s->whole = w;
+    if (cudaMemset(s->ws, 0, total) != cudaSuccess ||
+        cudaMemcpy(base + desc_off, descs.data(), sizeof(aio::ProjDesc) * n_projs, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess) {
+        step_free(s);
+        return fail(AIO_ERR_CUDA, "step workspace initialisation failed");
     }
     if (flags & AIO_STEP_GRAPH) {
         cudaStream_t cs = nullptr;
@@ -481,7 +530,20 @@ aio_status aio_decode_step(aio_step_t s, void* stream) {
 aio_status aio_decode_step_kernels(aio_step_t s, int* n_kernels) {
     aio_status st = valid_step(s);
     if (st != AIO_OK) return st;
-    if (n_kernels) *n_kernels = s->n;
+    if (n_kernels) *n_kernels = s->persistent ? 1 : s->n;
+    return AIO_OK;
+}
+
+aio_status aio_decode_step_reset(aio_step_t s) {
+    aio_status st = valid_step(s);
+    if (st != AIO_OK) return st;
+    if ((st = check_device(s->device)) != AIO_OK) return st;
+    const size_t desc_off = reinterpret_cast<const uint8_t*>(s->whole.projs) - static_cast<const uint8_t*>(s->ws);
+    const size_t done_off = reinterpret_cast<const uint8_t*>(s->whole.done) - static_cast<const uint8_t*>(s->ws);
+    AIO_CUDA(cudaDeviceSynchronize());
+    AIO_CUDA(cudaMemset(s->ws, 0, desc_off));   // partial sums and tile counters
+    AIO_CUDA(cudaMemset(static_cast<uint8_t*>(s->ws) + done_off, 0, s->ws_bytes - done_off));  // done, errors
+    AIO_CUDA(cudaDeviceSynchronize());
     return AIO_OK;
 }
 
@@ -512,7 +574,7 @@ aio_status aio_probe_read(const void* buf, size_t bytes, unsigned* out, void* st
     int dev = 0, sms = 0;
     aio_status st = current_device(&dev, &sms);
     if (st != AIO_OK) return st;
-    AIO_CUDA(aio::launch_probe(buf, static_cast<long long>(bytes / 4096), out, 2 * sms, static_cast<cudaStream_t>(stream)));
+    AIO_CUDA(aio::launch_probe(buf, static_cast<long long>(bytes / 4096), out, sms, static_cast<cudaStream_t>(stream)));
     return AIO_OK;
 }
 

@@ -1,29 +1,40 @@
-// aio_gemv.cu -- the decode-step linear kernel: y = x W^T for M = 1..8 token rows,
-// bf16 weights or int8 codes with per-output-channel bf16 scales (Sec. 2.1, Sec. 2.4).
+// aio_gemv.cu -- the decode-step stream kernel: y = x W^T for M = 1..8 token rows, bf16 weights or
+// int8 codes with per-output-channel bf16 scales (Sec. 2.1, Sec. 2.4), for one projection or for
+// every projection of a decode step in one persistent launch (Sec. 3.1).
 //
-// The work is a stream of weight bytes from HBM with 1 (bf16) or 2 (int8) FMAs per byte per
-// token row, so the kernel is built around keeping enough bytes in flight:
+// The work is a stream of weight bytes from HBM with 1 (bf16) or 2 (int8) multiply-adds per byte per
+// token row.  Design:
 //
-//   * Weights are cut into tiles of 8 rows x 256 k (4 KB bf16, 2 KB int8), each one contiguous
-//     block in the packed layout.  The T tiles of a matrix are split evenly over the Z warps of
-//     the grid: warp z streams tiles [z*T/Z, (z+1)*T/Z), so every warp (and CTA) moves the same
-//     number of bytes to within one tile, whatever N and K are.
-//   * Each warp owns a 12 KB ring in shared memory.  Lane 0 issues one cp.async.bulk per tile
-//     (global -> shared, L2 evict-first), completing on that slot's mbarrier; the warp waits on
-//     the mbarrier (bounded by %globaltimer), computes, and refills the slot.  No producer warp,
-//     no inter-warp synchronisation on the hot loop.
-//   * Lane j owns k-columns [8j, 8j+8) of every tile; it keeps 8 rows x M accumulators in
-//     registers and loads its 8 x values per row of x once per tile (reused by 8 weight rows).
-//     bf16 -> fp32 is a shift/mask; int8 -> fp32 is exact via a byte permute into the mantissa
-//     of 2^23 and one subtraction.  The int8 scale multiplies the finished fp32 sum.
-//   * A row group whose tiles all lie in one warp's segment is reduced across lanes (shuffles)
-//     and written directly.  A row group split between warps is finished by the last warp to
-//     add its tile count to the group's counter: every contributor stores its partial sums,
-//     fences, and bumps the counter; the last one sums all partials in warp order (so the
-//     result is deterministic), writes y and resets the counter to zero.  Nothing spins.
-//   * Programmatic dependent launch: the kernel signals its dependents at entry and issues its
-//     first weight copies before griddepcontrol.wait, so it prefetches W while the previous
-//     kernel on the stream finishes; x, y and the workspace are touched only after the wait.
+//   * Tiles.  W is cut into tiles of 8 rows x 256 k (4 KB bf16, 2 KB int8); consecutive tiles are
+//     contiguous in the packed layout, so any run of them is one bulk copy.  The T tiles of a matrix
+//     are split evenly over the Z warps of the grid: warp z streams tiles [z*T/Z, (z+1)*T/Z), so
+//     every warp moves the same bytes to within one tile whatever N and K are.
+//   * Rings.  One CTA per SM; each warp owns a shared-memory ring of slots.  Lane 0 issues one
+//     cp.async.bulk per slot (global -> shared, L2 evict-first) completing on the slot's mbarrier;
+//     the warp waits (bounded by %globaltimer), computes, and refills the slot.  The issue cursor
+//     runs ahead across projection boundaries: weights never depend on x.
+//   * Arithmetic on the tensor cores.  For the 16-k step s of a tile, lane (g, c) = (lane/4, lane%4)
+//     supplies x[token g][64c + 4s + 0..3] as its A fragment (rows 8..15 of A are zero) and
+//     W[row g][64c + 4s + 0..3] as its B fragment of one mma.sync.m16n8k16 (bf16 in, fp32
+//     accumulate).  This assignment of the 256 k of a tile to (s, c, position) is a permutation
+//     shared by A and B, so the sum is unchanged; it makes each lane's 64 W elements and 64 x
+//     elements of a tile contiguous.  Full tiles are stored in fragment order ([j][lane][16 B]),
+//     so the W loads are conflict-free 128-bit shared loads.  D[token g][row 2c, 2c+1] lands in
+//     lane (g, c): the k-reduction across lanes is done by the MMA, and the work per byte does not
+//     grow with M.  k-step s accumulates into one of four chains (s % 4) to keep MMAs in flight.
+//     int8 codes become bf16 exactly (|q| <= 128 fits bf16's 8 significant bits) with two bit
+//     operations and one bf16x2 subtraction per pair; the per-channel scale multiplies the
+//     finished fp32 sum.
+//   * Split row groups.  A row group whose tiles all lie in one warp's segment is written directly.
+//     One split between warps is finished by the last warp to add its tile count to the group's
+//     counter: contributors store partial sums, fence, count; the last one sums the partials in
+//     warp order (deterministic), writes y and resets the counter.  Nothing spins.
+//   * Projection order.  In a persistent step, projection p+1 reads x only after every CTA has
+//     finished projection p: warps count in shared memory, the last warp of a CTA makes one global
+//     increment, warp 0 of each CTA polls the global counter (bounded) and publishes it to its CTA.
+//   * Programmatic dependent launch: the kernel signals dependents at entry and issues its first
+//     weight copies before griddepcontrol.wait; x, y and the workspace are touched after it.
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -98,27 +109,49 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
-// ------------------------------------------------------------------ element helpers
-__device__ __forceinline__ void bf16x8_to_f32(const uint4 v, float (&f)[8]) {
-    f[0] = __uint_as_float(v.x << 16); f[1] = __uint_as_float(v.x & 0xFFFF0000u);
-    f[2] = __uint_as_float(v.y << 16); f[3] = __uint_as_float(v.y & 0xFFFF0000u);
-    f[4] = __uint_as_float(v.z << 16); f[5] = __uint_as_float(v.z & 0xFFFF0000u);
-    f[6] = __uint_as_float(v.w << 16); f[7] = __uint_as_float(v.w & 0xFFFF0000u);
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
 
-// int8 codes -> exact fp32.  (q ^ 0x80) is q + 128 as an unsigned byte u; placed in the low
-// mantissa byte of 2^23 it reads as 2^23 + u, and subtracting 2^23 + 128 gives q exactly.
-__device__ __forceinline__ void i8x8_to_f32(const uint2 v, float (&f)[8]) {
-    const uint32_t a = v.x ^ 0x80808080u, b = v.y ^ 0x80808080u;
-    const float bias = 8388736.0f;  // 2^23 + 128
-    f[0] = __uint_as_float(__byte_perm(a, 0x4B000000u, 0x7440)) - bias;
-    f[1] = __uint_as_float(__byte_perm(a, 0x4B000000u, 0x7441)) - bias;
-    f[2] = __uint_as_float(__byte_perm(a, 0x4B000000u, 0x7442)) - bias;
-    f[3] = __uint_as_float(__byte_perm(a, 0x4B000000u, 0x7443)) - bias;
-    f[4] = __uint_as_float(__byte_perm(b, 0x4B000000u, 0x7440)) - bias;
-    f[5] = __uint_as_float(__byte_perm(b, 0x4B000000u, 0x7441)) - bias;
-    f[6] = __uint_as_float(__byte_perm(b, 0x4B000000u, 0x7442)) - bias;
-    f[7] = __uint_as_float(__byte_perm(b, 0x4B000000u, 0x7443)) - bias;
+__device__ __forceinline__ unsigned ld_acquire_cta_shared(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(smem_addr(p)) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_release_cta_shared(unsigned* p, unsigned v) {
+    asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(smem_addr(p)), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ unsigned atom_add_acq_rel_cta_shared(unsigned* p, unsigned v) {
+    unsigned old;
+    asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], %2;" : "=r"(old) : "r"(smem_addr(p)), "r"(v) : "memory");
+    return old;
+}
+
+// D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Two int8 codes (the bytes of w selected by SEL) -> bf16x2, exactly.  With t holding the code bytes
+// in the low byte of each 16-bit half: 0x4300 | (q & 0x7F) is bf16 128 + (q & 0x7F), and
+// 0x4300 | (q & 0x80) is bf16 128 or 256; their difference is q.
+template <uint32_t SEL>
+__device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t w) {
+    const uint32_t t = __byte_perm(w, 0u, SEL);
+    const uint32_t a = (t & 0x007F007Fu) | 0x43004300u;
+    const uint32_t b = (t & 0x00800080u) | 0x43004300u;
+    __nv_bfloat162 r = __hsub2(*reinterpret_cast<const __nv_bfloat162*>(&a),
+                               *reinterpret_cast<const __nv_bfloat162*>(&b));
+    return *reinterpret_cast<uint32_t*>(&r);
 }
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
@@ -126,289 +159,573 @@ __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_floa
 template <bool I8>
 struct TileT {
     static constexpr int kEsize = I8 ? 1 : 2;
-    static constexpr int kBytes = kRows * kKT * kEsize;       // 2048 or 4096
-    static constexpr int kStages = kRingBytesPerWarp / kBytes;  // 6 or 3
-    static_assert(kStages <= kMaxStages, "ring slots exceed the barrier area");
+    static constexpr int kBytes = kRows * kKT * kEsize;    // 2048 or 4096
+    static constexpr int kChunk = kSlotBytes / kBytes;     // tiles per ring slot
+    static constexpr int kPieces = kBytes / 512;           // 16-byte pieces per lane per tile (4 or 8)
+    static constexpr int kPieceElems = 16 / kEsize;        // elements per piece (16 or 8)
 };
 
-struct TileCoord {
-    int g, kt, rows, klen;
-};
-
-__device__ __forceinline__ TileCoord tile_coord(const GemvArgs& a, long long t) {
-    TileCoord c;
-    c.g = static_cast<int>(t / a.NKT);
-    c.kt = static_cast<int>(t - static_cast<long long>(c.g) * a.NKT);
-    c.rows = min(kRows, a.N - c.g * kRows);
-    c.klen = min(kKT, a.K - c.kt * kKT);
-    return c;
+__device__ __forceinline__ const ProjDesc* proj_desc(const StreamArgs& s, int p) {
+    return s.projs ? s.projs + p : &s.one;
 }
 
-// Lane 0: arm the slot's barrier with the tile's byte count and issue its bulk copy (or, for
-// row-major weights, one copy per row of the tile).
+// Byte offset of tile (g, kt) in the packed layout.
+template <int E>
+__device__ __forceinline__ size_t tile_offset(int K, int N, int g, int kt) {
+    const int rows = min(kRows, N - g * kRows);
+    return (static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT) * E;
+}
+
+// Lane 0: arm the slot's barrier with the chunk's byte count and issue the copies of tiles
+// [t, t + nt) of projection d.  Packed weights: one bulk copy.  Row-major weights: one copy per
+// tile row, landing in the row-major form of that tile.
 template <bool I8>
-__device__ __forceinline__ void issue_tile(const GemvArgs& a, long long t, uint8_t* dst, uint64_t* bar,
-                                           uint64_t pol) {
+__device__ __noinline__ void issue_chunk_general(const ProjDesc* d, int t, int nt, uint8_t* dst, uint64_t* bar,
+                                                 uint64_t pol) {
     constexpr int E = TileT<I8>::kEsize;
-    const TileCoord c = tile_coord(a, t);
-    const uint32_t bytes = static_cast<uint32_t>(c.rows * c.klen * E);
-    mbar_expect_tx(bar, bytes);
-    if (!a.rowmajor) {
-        const size_t off = (static_cast<size_t>(c.g) * kRows * a.K + static_cast<size_t>(c.kt) * c.rows * kKT) * E;
-        bulk_g2s(dst, a.w + off, bytes, bar, pol);
-    } else {
-        for (int r = 0; r < c.rows; ++r) {
-            const size_t off = (static_cast<size_t>(c.g * kRows + r) * a.K + static_cast<size_t>(c.kt) * kKT) * E;
-            bulk_g2s(dst + r * c.klen * E, a.w + off, static_cast<uint32_t>(c.klen * E), bar, pol);
+    const int K = d->K, N = d->N, NKT = d->NKT;
+    int g = t / NKT, kt = t - g * NKT;
+    if (!d->rowmajor) {
+        const int tl = t + nt - 1;
+        const int gl = tl / NKT, ktl = tl - gl * NKT;
+        const int rows_l = min(kRows, N - gl * kRows), klen_l = min(kKT, K - ktl * kKT);
+        const size_t off = tile_offset<E>(K, N, g, kt);
+        const size_t end = tile_offset<E>(K, N, gl, ktl) + static_cast<size_t>(rows_l) * klen_l * E;
+        const uint32_t bytes = static_cast<uint32_t>(end - off);
+        mbar_expect_tx(bar, bytes);
+        bulk_g2s(dst, d->w + off, bytes, bar, pol);
+        return;
+    }
+    uint32_t total = 0;
+    {
+        int gg = g, kk = kt;
+        for (int j = 0; j < nt; ++j) {
+            total += static_cast<uint32_t>(min(kRows, N - gg * kRows) * min(kKT, K - kk * kKT) * E);
+            if (++kk == NKT) { kk = 0; ++gg; }
         }
     }
-}
-
-// acc[r][m] += sum over this lane's 8 columns of W[row r] * x[m]
-template <int MT, bool I8>
-__device__ __forceinline__ void tile_fma(float (&acc)[kRows][MT], const uint8_t* tile, const TileCoord& c,
-                                         int lane, const GemvArgs& a) {
-    constexpr int E = TileT<I8>::kEsize;
-    if (lane * 8 >= c.klen) return;
-    float xf[MT][8];
-    const uint16_t* xp = a.x + static_cast<size_t>(c.kt) * kKT + lane * 8;
-#pragma unroll
-    for (int m = 0; m < MT; ++m) {
-        const uint4 v = *reinterpret_cast<const uint4*>(xp + static_cast<size_t>(m) * a.K);
-        bf16x8_to_f32(v, xf[m]);
-    }
-    const uint8_t* base = tile + lane * 8 * E;
-#pragma unroll
-    for (int r = 0; r < kRows; ++r) {
-        if (r < c.rows) {
-            float wf[8];
-            if constexpr (I8) {
-                i8x8_to_f32(*reinterpret_cast<const uint2*>(base + r * c.klen), wf);
-            } else {
-                bf16x8_to_f32(*reinterpret_cast<const uint4*>(base + r * c.klen * 2), wf);
-            }
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[r][m] = fmaf(wf[e], xf[m][e], acc[r][m]);
-            }
+    mbar_expect_tx(bar, total);
+    for (int j = 0; j < nt; ++j) {
+        const int rows = min(kRows, N - g * kRows), klen = min(kKT, K - kt * kKT);
+        for (int r = 0; r < rows; ++r) {
+            const size_t off = (static_cast<size_t>(g * kRows + r) * K + static_cast<size_t>(kt) * kKT) * E;
+            bulk_g2s(dst + r * klen * E, d->w + off, static_cast<uint32_t>(klen * E), bar, pol);
         }
+        dst += rows * klen * E;
+        if (++kt == NKT) { kt = 0; ++g; }
     }
 }
 
 template <bool I8>
-__device__ __forceinline__ float row_scale(const GemvArgs& a, int n) {
+__device__ __forceinline__ void issue_chunk(const ProjDesc* d, int t, int nt, uint8_t* dst, uint64_t* bar,
+                                            uint64_t pol) {
+    constexpr int B = TileT<I8>::kBytes;
+    if (d->uniform) {   // every tile full: tile t is bytes [t * B, (t + 1) * B)
+        const uint32_t bytes = static_cast<uint32_t>(nt * B);
+        mbar_expect_tx(bar, bytes);
+        bulk_g2s(dst, d->w + static_cast<size_t>(t) * B, bytes, bar, pol);
+        return;
+    }
+    issue_chunk_general<I8>(d, t, nt, dst, bar, pol);
+}
+
+// A warp's walk over its tiles of every projection, one chunk (<= C consecutive tiles) at a time.
+struct ChunkCursor {
+    int p, t, te;
+};
+
+__device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, long long z, int Z) {
+    const long long T = proj_desc(s, 0)->T;
+    c.p = 0;
+    c.t = static_cast<int>(z * T / Z);
+    c.te = static_cast<int>((z + 1) * T / Z);
+}
+
+// Next chunk of the walk: its projection, first tile and tile count; false at the end.
+__device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s, long long z, int Z, int C, int& p,
+                                            int& t, int& nt) {
+    while (c.t >= c.te) {
+        if (c.p + 1 >= s.nproj) return false;
+        ++c.p;
+        const long long T = proj_desc(s, c.p)->T;
+        c.t = static_cast<int>(z * T / Z);
+        c.te = static_cast<int>((z + 1) * T / Z);
+    }
+    p = c.p;
+    t = c.t;
+    nt = min(C, c.te - c.t);
+    c.t += nt;
+    return true;
+}
+
+// The fields of one projection the consuming warp needs, held in registers.
+struct Proj {
+    const uint16_t* x;
+    const uint16_t* scales;
+    float* y;
+    float* partial;
+    unsigned* counters;
+    long long T;
+    int M, K, N, NKT;
+    int rowmajor, uniform;
+};
+
+__device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
+    Proj p;
+    p.x = d->x;
+    p.scales = d->scales;
+    p.y = d->y;
+    p.partial = d->partial;
+    p.counters = d->counters;
+    p.T = d->T;
+    p.M = M;
+    p.K = d->K;
+    p.N = d->N;
+    p.NKT = d->NKT;
+    p.rowmajor = d->rowmajor;
+    p.uniform = d->uniform;
+    return p;
+}
+
+// One tile: D += x[:, k-range] * W[rows, k-range]^T on the tensor cores.  Lane (g, c) loads its 16
+// k-steps' worth of W (row g) and x (token g), each 64 contiguous k starting at 64c.  Full packed
+// tiles use the fragment-ordered layout; ragged tiles (rows < 8 or klen < 256) and row-major
+// weights are row-major, and any piece outside the tile (or a token >= M) is zero.  k-step s
+// accumulates into d[s % 4], so four MMA chains are in flight instead of one.
+template <bool I8>
+__device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, int rows, int klen, int kbase,
+                                         int lane, const Proj& P) {
+    using TL = TileT<I8>;
+    constexpr int NP = TL::kPieces;          // 16-byte W pieces per lane
+    constexpr int PE = TL::kPieceElems;      // elements per W piece
+    const int g = lane >> 2, c = lane & 3;
+    const bool full = rows == kRows && klen == kKT && !P.rowmajor;
+    uint4 w[NP];
+#pragma unroll
+    for (int j = 0; j < NP; ++j) {
+        if (full) {
+            w[j] = *reinterpret_cast<const uint4*>(tile + j * 512 + lane * 16);
+        } else {
+            const int k = 64 * c + PE * j;
+            if (g < rows && k < klen)
+                w[j] = *reinterpret_cast<const uint4*>(tile + (static_cast<size_t>(g) * klen + k) * TL::kEsize);
+            else
+                w[j] = make_uint4(0u, 0u, 0u, 0u);
+        }
+    }
+    // x: 64 bf16 of token g starting at kbase + 64c, as 8 pieces of 8
+    uint4 xv[8];
+    const bool xrow = g < P.M;
+    const uint16_t* xp = P.x + static_cast<size_t>(g) * P.K + kbase + 64 * c;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (xrow && 64 * c + 8 * j < klen)
+            xv[j] = *reinterpret_cast<const uint4*>(xp + 8 * j);
+        else
+            xv[j] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    // k-step s covers elements 4s..4s+3 of the lane's 64: x piece s/2, words 2(s%2), 2(s%2)+1
+#pragma unroll
+    for (int s = 0; s < 16; ++s) {
+        const uint4& xq = xv[s >> 1];
+        const uint32_t a0 = (s & 1) ? xq.z : xq.x;
+        const uint32_t a2 = (s & 1) ? xq.w : xq.y;
+        uint32_t b0, b1;
+        if constexpr (I8) {
+            // W piece s/4 holds codes 16*(s/4) .. +15; k-step s uses word s%4 (4 codes)
+            const uint4& wq = w[s >> 2];
+            const uint32_t word = (s & 3) == 0 ? wq.x : (s & 3) == 1 ? wq.y : (s & 3) == 2 ? wq.z : wq.w;
+            b0 = i8x2_to_bf16x2<0x4140u>(word);
+            b1 = i8x2_to_bf16x2<0x4342u>(word);
+        } else {
+            const uint4& wq = w[s >> 1];
+            b0 = (s & 1) ? wq.z : wq.x;
+            b1 = (s & 1) ? wq.w : wq.y;
+        }
+        mma_bf16(d[s & 3], a0, 0u, a2, 0u, b0, b1);
+    }
+}
+
+// The same for a full packed tile, with no bounds logic: W pieces at j * 512 + lane * 16 of the
+// tile, x pieces at xp + 8j (xp = x + token * K + 256 kt + 64c), x zero for tokens >= M.
+template <bool I8>
+__device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp,
+                                              bool xrow) {
+    using TL = TileT<I8>;
+    constexpr int NP = TL::kPieces;
+    uint4 w[NP];
+#pragma unroll
+    for (int j = 0; j < NP; ++j) w[j] = *reinterpret_cast<const uint4*>(tile_lane + j * 512);
+    uint4 xv[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+        xv[j] = xrow ? *reinterpret_cast<const uint4*>(xp + 8 * j) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int s = 0; s < 16; ++s) {
+        const uint4& xq = xv[s >> 1];
+        const uint32_t a0 = (s & 1) ? xq.z : xq.x;
+        const uint32_t a2 = (s & 1) ? xq.w : xq.y;
+        uint32_t b0, b1;
+        if constexpr (I8) {
+            const uint4& wq = w[s >> 2];
+            const uint32_t word = (s & 3) == 0 ? wq.x : (s & 3) == 1 ? wq.y : (s & 3) == 2 ? wq.z : wq.w;
+            b0 = i8x2_to_bf16x2<0x4140u>(word);
+            b1 = i8x2_to_bf16x2<0x4342u>(word);
+        } else {
+            const uint4& wq = w[s >> 1];
+            b0 = (s & 1) ? wq.z : wq.x;
+            b1 = (s & 1) ? wq.w : wq.y;
+        }
+        mma_bf16(d[s & 3], a0, 0u, a2, 0u, b0, b1);
+    }
+}
+
+template <bool I8>
+__device__ __forceinline__ float row_scale(const Proj& P, int n) {
     if constexpr (I8) {
-        return bf16_to_f32(a.scales[n]);
+        return bf16_to_f32(P.scales[n]);
     } else {
         return 1.0f;
     }
 }
 
-// Warp z has finished its tiles of row group g (kt in [kt_lo, kt_hi]): reduce over lanes and
-// either write y (group complete in this warp) or hand the partial to the last-arriver fixup.
-template <int MT, bool I8>
-__device__ __forceinline__ void finish_group(const GemvArgs& a, float (&acc)[kRows][MT], const TileCoord& c,
-                                             long long z, long long t0, long long t1, int lane) {
-#pragma unroll
-    for (int r = 0; r < kRows; ++r) {
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-            float v = acc[r][m];
-            v += __shfl_xor_sync(0xffffffffu, v, 16);
-            v += __shfl_xor_sync(0xffffffffu, v, 8);
-            v += __shfl_xor_sync(0xffffffffu, v, 4);
-            v += __shfl_xor_sync(0xffffffffu, v, 2);
-            v += __shfl_xor_sync(0xffffffffu, v, 1);
-            acc[r][m] = v;
-        }
-    }
-    const long long gfirst = static_cast<long long>(c.g) * a.NKT;
+// Warp z has finished its tiles of row group g: lane (g', c) holds D[token g'][rows 2c, 2c+1].
+// Write y (group complete in this warp) or hand the partial to the last-arriver fixup.
+template <bool I8>
+__device__ __forceinline__ void finish_group(const Proj& P, int Z, const float (&d)[4], int g, int rows, long long z,
+                                             long long t0, long long t1, int lane) {
+    const int tok = lane >> 2, r0 = 2 * (lane & 3);
+    const int row0 = g * kRows;
+    const long long gfirst = static_cast<long long>(g) * P.NKT;
     const int kt_lo = t0 > gfirst ? static_cast<int>(t0 - gfirst) : 0;
-    const int kt_hi = static_cast<int>(min(static_cast<long long>(a.NKT - 1), t1 - 1 - gfirst));
-    const int row0 = c.g * kRows;
+    const int kt_hi = static_cast<int>(min(static_cast<long long>(P.NKT - 1), t1 - 1 - gfirst));
+    const bool mine = tok < P.M;
 
-    if (kt_lo == 0 && kt_hi == a.NKT - 1) {
-#pragma unroll
-        for (int r = 0; r < kRows; ++r) {
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                if (((r * MT + m) & 31) == lane && r < c.rows)
-                    a.y[static_cast<size_t>(m) * a.N + row0 + r] = acc[r][m] * row_scale<I8>(a, row0 + r);
-            }
+    if (kt_lo == 0 && kt_hi == P.NKT - 1) {
+        if (mine) {
+            float* yp = P.y + static_cast<size_t>(tok) * P.N + row0 + r0;
+            if (r0 < rows) yp[0] = d[0] * row_scale<I8>(P, row0 + r0);
+            if (r0 + 1 < rows) yp[1] = d[1] * row_scale<I8>(P, row0 + r0 + 1);
         }
         return;
     }
 
-    // Split group: publish this warp's partial, then count tiles; the warp completing the
-    // count owns the final sum.
-    constexpr int V = kRows * MT;
-    const int side = (c.g == static_cast<int>(t0 / a.NKT)) ? 0 : 1;
-    float* mine = a.partial + (static_cast<size_t>(z) * 2 + side) * V;
-#pragma unroll
-    for (int r = 0; r < kRows; ++r) {
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-            if (((r * MT + m) & 31) == lane) mine[r * MT + m] = acc[r][m];
-        }
+    // Split group: publish this warp's partial [token][row], then count tiles; the warp completing
+    // the count owns the final sum.
+    const int V = kRows * P.M;
+    const int side = (g == static_cast<int>(t0 / P.NKT)) ? 0 : 1;
+    float* part = P.partial + (static_cast<size_t>(z) * 2 + side) * V;
+    if (mine) {
+        part[tok * kRows + r0] = d[0];
+        part[tok * kRows + r0 + 1] = d[1];
     }
     __threadfence();
     __syncwarp();
     const unsigned ntk = static_cast<unsigned>(kt_hi - kt_lo + 1);
     unsigned prev = 0;
-    if (lane == 0) prev = atomicAdd(&a.counters[c.g], ntk);
+    if (lane == 0) prev = atomicAdd(&P.counters[g], ntk);
     prev = __shfl_sync(0xffffffffu, prev, 0);
-    if (prev + ntk != static_cast<unsigned>(a.NKT)) return;
+    if (prev + ntk != static_cast<unsigned>(P.NKT)) return;
 
     __threadfence();
-    const long long tf = gfirst, tl = gfirst + a.NKT - 1;
-    const long long zf = ((tf + 1) * a.Z - 1) / a.T;   // warp whose segment holds tile tf
-    const long long zl = ((tl + 1) * a.Z - 1) / a.T;   // ... and tile tl
+    const long long tf = gfirst, tl = gfirst + P.NKT - 1;
+    const long long zf = ((tf + 1) * Z - 1) / P.T;   // warp whose segment holds tile tf
+    const long long zl = ((tl + 1) * Z - 1) / P.T;   // ... and tile tl
     for (int v = lane; v < V; v += 32) {
-        const int r = v / MT, m = v - (v / MT) * MT;
-        if (r >= c.rows) continue;
+        const int m = v / kRows, r = v - m * kRows;
+        if (r >= rows) continue;
         float sum = 0.0f;
         for (long long zz = zf; zz <= zl; ++zz) {
-            const long long s0 = zz * a.T / a.Z, s1 = (zz + 1) * a.T / a.Z;
+            const long long s0 = zz * P.T / Z, s1 = (zz + 1) * P.T / Z;
             if (s1 == s0) continue;
-            const int sd = (c.g == static_cast<int>(s0 / a.NKT)) ? 0 : 1;
-            sum += __ldcg(a.partial + (static_cast<size_t>(zz) * 2 + sd) * V + v);
+            const int sd = (g == static_cast<int>(s0 / P.NKT)) ? 0 : 1;
+            sum += __ldcg(P.partial + (static_cast<size_t>(zz) * 2 + sd) * V + v);
         }
-        a.y[static_cast<size_t>(m) * a.N + row0 + r] = sum * row_scale<I8>(a, row0 + r);
+        P.y[static_cast<size_t>(m) * P.N + row0 + r] = sum * row_scale<I8>(P, row0 + r);
     }
-    if (lane == 0) a.counters[c.g] = 0u;
+    if (lane == 0) P.counters[g] = 0u;
 }
 
+// Lane 0 polls until *counter >= target (bounded by limit_ns); the result is broadcast to the warp.
+__device__ __noinline__ bool poll_global(const unsigned* counter, unsigned target, unsigned long long limit_ns,
+                                         int lane) {
+    int ok = 1;
+    if (lane == 0 && ld_acquire(counter) < target) {
+        const uint64_t start = globaltimer_ns();
+        while (ld_acquire(counter) < target) {
+            if (globaltimer_ns() - start > limit_ns) {
+                ok = 0;
+                break;
+            }
+        }
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+// Same for a CTA-local flag in shared memory.
+__device__ __noinline__ bool poll_shared(const unsigned* flag, unsigned target, unsigned long long limit_ns,
+                                         int lane) {
+    int ok = 1;
+    if (lane == 0 && ld_acquire_cta_shared(flag) < target) {
+        const uint64_t start = globaltimer_ns();
+        while (ld_acquire_cta_shared(flag) < target) {
+            if (globaltimer_ns() - start > limit_ns) {
+                ok = 0;
+                break;
+            }
+            __nanosleep(32);
+        }
+    }
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+// This warp has finished its part of a phase (a projection, or the whole kernel).  Warps count in
+// shared memory with acquire-release semantics; the last warp of the CTA fences at device scope
+// (cumulatively publishing what every warp of the CTA wrote in the phase) and makes the one global
+// increment.  Returns the global counter's previous value in the last warp, ~0u elsewhere.
+__device__ __forceinline__ unsigned cta_arrive(unsigned* cta_count, unsigned* global_count, int lane) {
+    __syncwarp();
+    unsigned g = 0xffffffffu;
+    if (lane == 0) {
+        if (atom_add_acq_rel_cta_shared(cta_count, 1u) == static_cast<unsigned>(kWarps - 1)) {
+            *cta_count = 0u;   // no warp of this CTA can arrive again before this phase completes
+            __threadfence();
+            g = atomicAdd(global_count, 1u);
+        }
+    }
+    return __shfl_sync(0xffffffffu, g, 0);
+}
+
+// The stream kernel: one CTA per SM, every warp streams its segment of every projection through
+// its own bulk-copy ring.  All per-tile bookkeeping is incremental 32-bit arithmetic; divisions
+// happen once per chunk (issue) or once per projection (consume).
 template <int MT, bool I8>
-__global__ void __launch_bounds__(kThreads, (MT <= 4) ? 2 : 1) aio_gemv_kernel(const GemvArgs a) {
+__global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_constant__ StreamArgs s) {
     using TL = TileT<I8>;
+    constexpr int C = TL::kChunk;
+    constexpr int S = kStages;
+    constexpr int E = TL::kEsize;
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     uint8_t* ring = smem + warp * kRingBytesPerWarp;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kRingBytesPerWarp) + warp * kMaxStages;
+    // CTA-level sync words: [0] warps of this CTA done with the current phase, [1] highest projection
+    // index whose predecessor is known complete (published by warp 0).
+    unsigned* cta_sync = reinterpret_cast<unsigned*>(smem + kSyncOffset);
 
     griddep_launch_dependents();
 
     const long long z = static_cast<long long>(blockIdx.x) * kWarps + warp;
-    const long long t0 = z * a.T / a.Z;
-    const long long t1 = (z + 1) * a.T / a.Z;
-    const int ntiles = static_cast<int>(t1 - t0);
-
+    const int Z = s.Z;
     if (lane == 0) {
 #pragma unroll
-        for (int s = 0; s < TL::kStages; ++s) mbar_init(&bars[s], 1);
+        for (int i = 0; i < S; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
-    __syncwarp();
-
+    if (threadIdx.x == 0) {
+        cta_sync[0] = 0u;
+        cta_sync[1] = 0u;
+    }
+    __syncthreads();   // the only CTA-wide barrier: barriers and sync words are initialised
     const uint64_t pol = policy_evict_first();
-    const bool stall = a.test_stall && z == a.Z - 1;  // the grid's last warp always owns >= 1 tile
-    if (lane == 0) {
-        const int npro = min(ntiles, TL::kStages);
-        for (int i = 0; i < npro; ++i) {
-            if (stall && i == 0) continue;  // test hook: this slot's barrier never completes
-            issue_tile<I8>(a, t0 + i, ring + i * TL::kBytes, &bars[i], pol);
-        }
+
+    // The issue cursor walks this warp's tiles of all projections in consumption order.
+    ChunkCursor ring_cur;
+    cursor_init(ring_cur, s, z, Z);
+    int islot = 0;
+    bool first_issue = true;
+    const bool stall = s.test_stall && z == Z - 1;   // the grid's last warp always owns >= 1 tile
+    auto issue_next = [&]() -> bool {
+        int ip, it, nt;
+        if (!cursor_next(ring_cur, s, z, Z, C, ip, it, nt)) return false;
+        if (lane == 0 && !(stall && first_issue))   // test hook: this slot's barrier never completes
+            issue_chunk<I8>(proj_desc(s, ip), it, nt, ring + islot * kSlotBytes, &bars[islot], pol);
+        first_issue = false;
+        islot = (islot + 1 == S) ? 0 : islot + 1;
+        return true;
+    };
+    int in_flight = 0;
+    for (int i = 0; i < S; ++i) {
+        if (!issue_next()) break;
+        ++in_flight;
     }
 
-    // Everything below reads x / writes y and the workspace: wait for the previous grid.
+    // With programmatic dependent launch, everything below (x, y, workspace) waits for the
+    // previous grid on the stream.
     griddep_wait();
 
-    float acc[kRows][MT];
-#pragma unroll
-    for (int r = 0; r < kRows; ++r)
-#pragma unroll
-        for (int m = 0; m < MT; ++m) acc[r][m] = 0.0f;
-
-    for (int i = 0; i < ntiles; ++i) {
-        const long long t = t0 + i;
-        const int s = i % TL::kStages;
-        const uint32_t parity = static_cast<uint32_t>(i / TL::kStages) & 1u;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&bars[s], parity, a.wait_limit_ns));
-        if (!ok) {
-            // Record the timeout, then wait (bounded) for this warp's other copies in flight so
-            // no bulk copy targets shared memory after the CTA exits.
-            if (lane == 0) atomicExch(a.err, kDevErrTimeout);
-            const int last_issued = min(ntiles, i + TL::kStages);
-            for (int j = i; j < last_issued; ++j)
-                mbar_wait(&bars[j % TL::kStages], static_cast<uint32_t>(j / TL::kStages) & 1u, a.wait_limit_ns);
-            return;
+    const unsigned G = gridDim.x;
+    int cslot = 0;
+    uint32_t cphase = 0;
+    bool dead = false;    // set after a timeout: stop consuming, keep signalling
+    for (int p = 0; p < s.nproj; ++p) {
+        const Proj P = load_proj(proj_desc(s, p), MT);
+        const long long t0 = z * P.T / Z, t1 = (z + 1) * P.T / Z;
+        if (p > 0) {
+            // Projection p reads x only after every CTA finished projection p-1.
+            bool ok;
+            if (warp == 0) {
+                const bool polled = !dead && poll_global(&s.done[p - 1], G, s.wait_limit_ns, lane);
+                ok = dead || polled;
+                if (lane == 0) st_release_cta_shared(&cta_sync[1], static_cast<unsigned>(p));
+                if (polled && p > 1 && blockIdx.x == 0 && lane == 0) s.done[p - 2] = 0u;   // nobody polls it any more
+            } else {
+                ok = poll_shared(&cta_sync[1], static_cast<unsigned>(p), s.wait_limit_ns, lane);
+            }
+            __syncwarp();
+            if (!ok && !dead) {
+                if (lane == 0) atomicExch(s.err, kDevErrGridTimeout);
+                dead = true;
+            }
         }
-        const TileCoord c = tile_coord(a, t);
-        tile_fma<MT, I8>(acc, ring + s * TL::kBytes, c, lane, a);
-        __syncwarp();
-        if (lane == 0 && i + TL::kStages < ntiles) {
-            fence_proxy_async_smem();  // order this warp's reads of the slot before the refill
-            issue_tile<I8>(a, t + TL::kStages, ring + s * TL::kBytes, &bars[s], pol);
+        if (!dead && t1 > t0) {
+            float d[4][4] = {};
+            const int NKT = P.NKT;
+            const int last_len = P.K - (NKT - 1) * kKT;
+            int t = static_cast<int>(t0);
+            const int tend = static_cast<int>(t1);
+            int g = t / NKT, kt = t - g * NKT;
+            int rows = min(kRows, P.N - g * kRows);
+            const bool xrow = (lane >> 2) < MT;
+            const uint16_t* xlane = P.x + static_cast<size_t>(lane >> 2) * P.K + 64 * (lane & 3);
+            while (t < tend) {
+                if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
+                    if (lane == 0) atomicExch(s.err, kDevErrTimeout);
+                    dead = true;
+                    break;
+                }
+                const int nt = min(C, tend - t);
+                const uint8_t* tp = ring + cslot * kSlotBytes;
+#pragma unroll
+                for (int j = 0; j < C; ++j) {
+                    if (j < nt) {
+                        const int klen = kt == NKT - 1 ? last_len : kKT;
+                        if (P.uniform) {
+                            tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, xrow);
+                        } else {
+                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P);
+                        }
+                        tp += rows * klen * E;
+                        if (kt == NKT - 1 || t == tend - 1) {
+                            float sum[4];
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
+                            finish_group<I8>(P, Z, sum, g, rows, z, t0, t1, lane);
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) d[q][i] = 0.0f;
+                        }
+                        ++t;
+                        if (++kt == NKT) {
+                            kt = 0;
+                            ++g;
+                            rows = min(kRows, P.N - g * kRows);
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) fence_proxy_async_smem();   // this warp's reads of the slot precede its refill
+                cslot = (cslot + 1 == S) ? 0 : cslot + 1;
+                cphase ^= (cslot == 0) ? 1u : 0u;
+                if (!issue_next()) --in_flight;
+            }
+            if (dead) {
+                // wait (bounded) for this warp's copies still in flight, then stop issuing
+                for (int j = 0; j < in_flight; ++j) {
+                    mbar_wait(&bars[cslot], cphase, s.wait_limit_ns);
+                    cslot = (cslot + 1 == S) ? 0 : cslot + 1;
+                    cphase ^= (cslot == 0) ? 1u : 0u;
+                }
+                in_flight = 0;
+            }
         }
-        if (c.kt == a.NKT - 1 || i == ntiles - 1) {
-            finish_group<MT, I8>(a, acc, c, z, t0, t1, lane);
-#pragma unroll
-            for (int r = 0; r < kRows; ++r)
-#pragma unroll
-                for (int m = 0; m < MT; ++m) acc[r][m] = 0.0f;
+        if (s.nproj > 1 && p + 1 < s.nproj) cta_arrive(&cta_sync[0], &s.done[p], lane);
+    }
+    if (s.nproj > 1) {
+        const unsigned prev = cta_arrive(&cta_sync[0], s.exit_count, lane);
+        if (lane == 0 && prev == G - 1) {
+            // every CTA has left: clear the counters no warp could clear while others might poll them
+            for (int q = max(0, s.nproj - 3); q < s.nproj; ++q) s.done[q] = 0u;
+            *s.exit_count = 0u;
         }
     }
 }
 
 // ------------------------------------------------------------------ read probe
-// Same per-warp ring as the linear kernel, 4 KB chunks, one word per chunk folded into *out.
-__global__ void __launch_bounds__(kThreads, 2) aio_probe_kernel(const uint8_t* buf, long long chunks, unsigned* out) {
-    constexpr int kChunk = 4096, kStages = kRingBytesPerWarp / kChunk;
+// Same per-warp ring and slot size as the stream kernel, no arithmetic: each warp streams a
+// contiguous range of 4 KB pages in slot-sized copies and folds word (lane * 32) of every page
+// into *out.  Measures the read ceiling of the bulk-copy ring.
+__global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* buf, long long pages, unsigned* out) {
+    constexpr int kPage = 4096, kPagesPerSlot = kSlotBytes / kPage;
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t* ring = smem + warp * kRingBytesPerWarp;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kRingBytesPerWarp) + warp * kMaxStages;
     const long long Z = static_cast<long long>(gridDim.x) * kWarps;
     const long long z = static_cast<long long>(blockIdx.x) * kWarps + warp;
-    const long long c0 = z * chunks / Z, c1 = (z + 1) * chunks / Z;
-    const int n = static_cast<int>(c1 - c0);
+    const long long p0 = z * pages / Z, p1 = (z + 1) * pages / Z;
     if (lane == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
+        for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     __syncwarp();
     const uint64_t pol = policy_evict_first();
-    if (lane == 0) {
-        for (int i = 0; i < min(n, kStages); ++i) {
-            mbar_expect_tx(&bars[i], kChunk);
-            bulk_g2s(ring + i * kChunk, buf + (c0 + i) * kChunk, kChunk, &bars[i], pol);
+    long long ip = p0;        // next page to issue
+    int islot = 0, in_flight = 0;
+    auto issue = [&]() -> bool {
+        if (ip >= p1) return false;
+        const int n = static_cast<int>(min(static_cast<long long>(kPagesPerSlot), p1 - ip));
+        if (lane == 0) {
+            mbar_expect_tx(&bars[islot], static_cast<uint32_t>(n * kPage));
+            bulk_g2s(ring + islot * kSlotBytes, buf + ip * kPage, static_cast<uint32_t>(n * kPage), &bars[islot], pol);
         }
-    }
+        ip += n;
+        islot = (islot + 1 == kStages) ? 0 : islot + 1;
+        return true;
+    };
+    for (int i = 0; i < kStages; ++i)
+        if (issue()) ++in_flight;
     unsigned acc = 0;
-    for (int i = 0; i < n; ++i) {
-        const int s = i % kStages;
-        if (!__all_sync(0xffffffffu, mbar_wait(&bars[s], static_cast<uint32_t>(i / kStages) & 1u, 1000000000ull))) {
-            for (int j = i + 1; j < min(n, i + kStages); ++j)
-                mbar_wait(&bars[j % kStages], static_cast<uint32_t>(j / kStages) & 1u, 1000000000ull);
+    int cslot = 0;
+    uint32_t cphase = 0;
+    for (long long pc = p0; pc < p1;) {
+        if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, 1000000000ull))) {
+            for (int j = 0; j < in_flight; ++j) {   // bounded drain of this warp's copies, then leave
+                mbar_wait(&bars[cslot], cphase, 1000000000ull);
+                cslot = (cslot + 1 == kStages) ? 0 : cslot + 1;
+                cphase ^= (cslot == 0) ? 1u : 0u;
+            }
             return;
         }
-        acc ^= reinterpret_cast<const unsigned*>(ring + s * kChunk)[lane * 32];
+        const int n = static_cast<int>(min(static_cast<long long>(kPagesPerSlot), p1 - pc));
+        for (int j = 0; j < n; ++j)
+            acc ^= reinterpret_cast<const unsigned*>(ring + cslot * kSlotBytes + j * kPage)[lane * 32];
+        pc += n;
         __syncwarp();
-        if (lane == 0 && i + kStages < n) {
-            fence_proxy_async_smem();
-            mbar_expect_tx(&bars[s], kChunk);
-            bulk_g2s(ring + s * kChunk, buf + (c0 + i + kStages) * kChunk, kChunk, &bars[s], pol);
-        }
+        if (lane == 0) fence_proxy_async_smem();
+        cslot = (cslot + 1 == kStages) ? 0 : cslot + 1;
+        cphase ^= (cslot == 0) ? 1u : 0u;
+        if (!issue()) --in_flight;
     }
     for (int o = 16; o; o >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, o);
     if (lane == 0) atomicXor(out, acc);
 }
 
-using GemvFn = void (*)(const GemvArgs);
+using StreamFn = void (*)(const StreamArgs);
 
 template <bool I8>
-GemvFn gemv_fn(int M) {
+StreamFn stream_fn(int M) {
     switch (M) {
-        case 1: return aio_gemv_kernel<1, I8>;
-        case 2: return aio_gemv_kernel<2, I8>;
-        case 3: return aio_gemv_kernel<3, I8>;
-        case 4: return aio_gemv_kernel<4, I8>;
-        case 5: return aio_gemv_kernel<5, I8>;
-        case 6: return aio_gemv_kernel<6, I8>;
-        case 7: return aio_gemv_kernel<7, I8>;
-        case 8: return aio_gemv_kernel<8, I8>;
+        case 1: return aio_stream_kernel<1, I8>;
+        case 2: return aio_stream_kernel<2, I8>;
+        case 3: return aio_stream_kernel<3, I8>;
+        case 4: return aio_stream_kernel<4, I8>;
+        case 5: return aio_stream_kernel<5, I8>;
+        case 6: return aio_stream_kernel<6, I8>;
+        case 7: return aio_stream_kernel<7, I8>;
+        case 8: return aio_stream_kernel<8, I8>;
         default: return nullptr;
     }
 }
@@ -418,7 +735,7 @@ GemvFn gemv_fn(int M) {
 cudaError_t prepare_kernels() {
     for (int i8 = 0; i8 < 2; ++i8) {
         for (int M = 1; M <= kMaxM; ++M) {
-            GemvFn f = i8 ? gemv_fn<true>(M) : gemv_fn<false>(M);
+            StreamFn f = i8 ? stream_fn<true>(M) : stream_fn<false>(M);
             cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
             if (e != cudaSuccess) return e;
         }
@@ -426,20 +743,35 @@ cudaError_t prepare_kernels() {
     return cudaFuncSetAttribute(aio_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
 }
 
-cudaError_t launch_gemv(const GemvArgs& a, bool i8, int grid, cudaStream_t s, bool pdl) {
-    GemvFn f = i8 ? gemv_fn<true>(a.M) : gemv_fn<false>(a.M);
+cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop) {
+    StreamFn f = i8 ? stream_fn<true>(a.M) : stream_fn<false>(a.M);
     if (!f) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(grid));
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = kSmemBytes;
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    int n = 0;
+    if (pdl) {
+        attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n].val.programmaticStreamSerializationAllowed = 1;
+        ++n;
+    }
+    if (coop) {
+        attr[n].id = cudaLaunchAttributeCooperative;
+        attr[n].val.cooperative = 1;
+        ++n;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
+    cfg.numAttrs = n;
     return cudaLaunchKernelEx(&cfg, f, a);
+}
+
+cudaError_t occupancy(bool i8, int M, int* blocks_per_sm) {
+    StreamFn f = i8 ? stream_fn<true>(M) : stream_fn<false>(M);
+    if (!f) return cudaErrorInvalidValue;
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, f, kThreads, kSmemBytes);
 }
 
 cudaError_t launch_probe(const void* buf, long long chunks, unsigned* out, int grid, cudaStream_t s) {

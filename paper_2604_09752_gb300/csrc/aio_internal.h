@@ -4,35 +4,65 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+// Build-time knobs (defaults are the shipped configuration).
+#ifndef AIO_RING_KB
+#define AIO_RING_KB 24          // shared-memory ring per warp, KB
+#endif
+#ifndef AIO_WARPS
+#define AIO_WARPS 8             // warps per CTA (one CTA per SM)
+#endif
+#ifndef AIO_SLOT_KB
+#define AIO_SLOT_KB 8           // bytes per ring slot, KB: one bulk copy of consecutive tiles
+#endif
+
 namespace aio {
 
 constexpr int kRows = 8;                    // rows per row group (AIO_ROWS_PER_GROUP)
 constexpr int kKT = 256;                    // k columns per tile (AIO_K_TILE)
-constexpr int kWarps = 8;                   // warps per CTA; every warp streams its own tile segment
+constexpr int kWarps = AIO_WARPS;           // every warp streams its own tile segment
 constexpr int kThreads = kWarps * 32;
-constexpr int kRingBytesPerWarp = 12 * 1024;  // per-warp shared-memory ring (3 bf16 tiles / 6 int8 tiles)
-constexpr int kMaxStages = 6;
-constexpr int kSmemBytes = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;
+constexpr int kRingBytesPerWarp = AIO_RING_KB * 1024;
+constexpr int kSlotBytes = AIO_SLOT_KB * 1024;
+constexpr int kStages = kRingBytesPerWarp / kSlotBytes;  // ring slots per warp
+constexpr int kMaxStages = kStages;
+static_assert(kSlotBytes % 4096 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
+constexpr int kSyncOffset = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;  // CTA-level sync words
+constexpr int kSmemBytes = kSyncOffset + 16;
 constexpr int kMaxM = 8;
+static_assert(kSmemBytes <= 227 * 1024, "ring does not fit in shared memory");
 
-constexpr int kDevErrTimeout = 1;
+constexpr int kDevErrTimeout = 1;       // a bulk-copy wait expired
+constexpr int kDevErrGridTimeout = 2;   // a wait for the previous projection expired
 
-// Everything one launch of the linear kernel needs.  Geometry:
-//   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles
-//   Z   = grid * kWarps warps; warp z streams tiles [z*T/Z, (z+1)*T/Z)
-struct GemvArgs {
+// One projection of a launch; read-only while the kernel runs.  Geometry:
+//   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles;
+//   warp z of the Z warps in the grid streams tiles [z*T/Z, (z+1)*T/Z) of every projection.
+struct ProjDesc {
     const uint16_t* x;        // [M, K] bf16
     const uint8_t* w;         // packed (or row-major) weights
     const uint16_t* scales;   // [N] bf16 (int8 only)
     float* y;                 // [M, N] fp32
     float* partial;           // [Z][2][kRows * M] partial sums of row groups split between warps
-    unsigned* counters;       // [NG] tiles accumulated so far per split row group; 0 between launches
-    int* err;                 // device error word
-    long long T;              // total tiles
-    int M, K, N;
-    int NG, NKT;
-    int Z;
+    unsigned* counters;       // [NG] tiles accumulated per split row group; zero between launches
+    long long T;
+    int K, N, NG, NKT;
     int rowmajor;             // 1: W is row-major [N, K]
+    int uniform;              // 1: packed, N % 8 == 0 and K % 256 == 0, so tile t is bytes [t, t+1) * tile size
+};
+static_assert(sizeof(ProjDesc) % 16 == 0, "descriptor array stride");
+
+// Kernel parameters.  A launch streams nproj projections back to back: projs[] in device memory,
+// or the single descriptor `one` when projs is null.  Projection p+1 reads its x only after every
+// CTA has finished projection p (done[p] == gridDim.x); done[] and the exit counter are zero at rest.
+struct StreamArgs {
+    const ProjDesc* projs;
+    ProjDesc one;
+    unsigned* done;           // [nproj] CTAs finished per projection (nproj > 1 only)
+    unsigned* exit_count;     // CTAs that have left the kernel (nproj > 1 only)
+    int* err;                 // device error word
+    int nproj;
+    int M;
+    int Z;
     int test_stall;           // 1: the grid's last warp skips its first copy (bounded-wait test)
     unsigned long long wait_limit_ns;
 };
@@ -43,11 +73,13 @@ struct Geometry {
 };
 
 Geometry geometry(int K, int N, int num_sms);
-size_t workspace_bytes(const Geometry& g, int M);   // partial + counters + error word, 256-B aligned parts
-void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters, int** err);
+size_t workspace_bytes(const Geometry& g, int M);   // partial sums + counters, 256-B aligned parts
+void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters);
 
 cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared memory)
-cudaError_t launch_gemv(const GemvArgs& a, bool i8, int grid, cudaStream_t s, bool pdl);
+// pdl: programmatic dependent launch; coop: cooperative launch (all CTAs co-resident).
+cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop);
+cudaError_t occupancy(bool i8, int M, int* blocks_per_sm);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
 cudaError_t launch_probe(const void* buf, long long chunks, unsigned* out, int grid, cudaStream_t s);
 

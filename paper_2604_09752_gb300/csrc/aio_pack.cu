@@ -1,9 +1,11 @@
-// aio_pack.cu -- weight packer: row-major W [N, K] <-> tiled layout (8 rows x 256 k tiles).
+// aio_pack.cu -- weight packer: row-major W [N, K] <-> tiled layout.
 //
-// The packed layout makes every tile one contiguous block so the linear kernel streams it with
-// a single bulk copy.  It is a pure permutation (no padding, bit-identical elements).  One
-// thread moves one 16-byte piece (8 bf16 or 16 int8 elements), which never straddles a tile
-// row because K % 16 == 0; reads of the row-major side are fully coalesced.
+// Tiles are 8 rows x 256 k; consecutive tiles are contiguous, so any run of them is one bulk copy.
+// A full tile (8 rows, 256 k) is stored in the order the stream kernel's lanes read it: 16-byte
+// piece j of lane L = 4 r + c holds W[row r][64 c + j * (8 bf16 | 16 int8) ...], at byte
+// j * 512 + L * 16 of the tile, so every 128-bit shared-memory load of a warp is contiguous.
+// Ragged tiles (last row group or last k tile) stay row-major.  The layout is a pure permutation
+// (no padding); one thread moves one 16-byte piece, and the row-major side is fully coalesced.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -26,13 +28,20 @@ __global__ void __launch_bounds__(256) aio_pack_kernel(const uint8_t* __restrict
         const int kt = k / kKT, kk = k - kt * kKT;
         const int rows = min(kRows, N - g * kRows);
         const int klen = min(kKT, K - kt * kKT);
-        const size_t packed = static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT +
-                              static_cast<size_t>(r) * klen + kk;
-        const size_t rowmajor = static_cast<size_t>(n) * K + k;
-        if (INVERSE) {
-            *reinterpret_cast<uint4*>(dst + rowmajor * E) = *reinterpret_cast<const uint4*>(src + packed * E);
+        const size_t tile = (static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT) * E;
+        size_t in_tile;
+        if (rows == kRows && klen == kKT) {
+            const int c = kk / 64, j = (kk - 64 * c) / kPiece;
+            in_tile = static_cast<size_t>(j) * 512 + (r * 4 + c) * 16;
         } else {
-            *reinterpret_cast<uint4*>(dst + packed * E) = *reinterpret_cast<const uint4*>(src + rowmajor * E);
+            in_tile = (static_cast<size_t>(r) * klen + kk) * E;
+        }
+        const size_t packed = tile + in_tile;
+        const size_t rowmajor = (static_cast<size_t>(n) * K + k) * E;
+        if (INVERSE) {
+            *reinterpret_cast<uint4*>(dst + rowmajor) = *reinterpret_cast<const uint4*>(src + packed);
+        } else {
+            *reinterpret_cast<uint4*>(dst + packed) = *reinterpret_cast<const uint4*>(src + rowmajor);
         }
     }
 }

@@ -1,0 +1,63 @@
+"""Run one projection (or one whole step) of a workload a few times: the small, self-contained case
+that profilers capture.
+
+  python -m paper_2604_09752_gb300.run_case --workload 7b-bf16 --proj lm_head --reps 3
+  python -m paper_2604_09752_gb300.run_case --workload 1b-bf16 --step --reps 3
+
+Prints the mean time per repetition from CUDA events.
+"""
+from __future__ import annotations
+
+import argparse
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--workload", default="7b-bf16")
+    ap.add_argument("--proj", default="lm_head", help="qkv, o, gate_up, down or lm_head (layer 0 / last)")
+    ap.add_argument("--M", type=int, default=1)
+    ap.add_argument("--step", action="store_true", help="run the whole decode step instead of one projection")
+    ap.add_argument("--layers", type=int, default=0, help="with --step: keep only this many layers (0 = all)")
+    ap.add_argument("--mode", choices=["persistent", "chain"], default="persistent")
+    ap.add_argument("--reps", type=int, default=3)
+    args = ap.parse_args()
+
+    import torch
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    from synth import workloads as swl
+
+    wl = swl.WORKLOADS[args.workload]
+    if args.step:
+        L = max(p.layer for p in wl.projs)
+        projs = [p for p in wl.projs if args.layers == 0 or p.layer < args.layers or p.layer == L]
+    else:
+        idx = swl.PROJ_NAMES.index(args.proj)
+        projs = [next(p for p in wl.projs if p.index == idx)]
+    dw = DeviceWorkload(wl, seed=0, max_M=args.M, projs=projs)
+    dw.fill_x(args.M)
+    flags = (aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT) if args.mode == "persistent" else \
+        (aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL)
+    run = (lambda: dw.step(args.M, flags)) if args.step else (lambda: dw.run_proj(0, args.M))
+    run()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.reps):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.reps
+    gb = dw.weight_bytes() / 1e9
+    print(f"{args.workload} {'step' if args.step else args.proj} M={args.M}: {ms:.4f} ms, {gb / ms * 1e3:.1f} GB/s")
+    dw.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -136,7 +136,7 @@ class DeviceWorkload:
         aio.aio_linear_run(b.handle, self.x_ptr(i), M, b.proj.K, b.proj.N, b.W.data_ptr(),
                            b.scales.data_ptr() if b.scales is not None else None, self.y_ptr(i), s)
 
-    def step_handle(self, M: int, flags: int = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL) -> int:
+    def step_handle(self, M: int, flags: int = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT) -> int:
         key = (M, flags)
         if key not in self._steps:
             projs = [(b.handle, self.x_ptr(i), b.W.data_ptr(),
@@ -145,7 +145,7 @@ class DeviceWorkload:
             self._steps[key] = aio.aio_decode_step_create(projs, M, flags)
         return self._steps[key]
 
-    def step(self, M: int, flags: int = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL, stream: Optional[int] = None):
+    def step(self, M: int, flags: int = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT, stream: Optional[int] = None):
         s = torch.cuda.current_stream(self.device).cuda_stream if stream is None else stream
         aio.aio_decode_step(self.step_handle(M, flags), s)
 

@@ -45,13 +45,14 @@ def test_small_step_graph_pdl(aio, name, M):
     dw = DeviceWorkload(swl.WORKLOADS[name], seed=1, max_M=8, projs=small_decoder(name))
     dw.fill_x(M)
     dw.step(M)
-    assert aio.aio_decode_step_kernels(dw.step_handle(M)) == len(dw.bufs)
+    assert aio.aio_decode_step_kernels(dw.step_handle(M)) == 1            # persistent: one launch
+    assert aio.aio_decode_step_kernels(dw.step_handle(M, aio.AIO_STEP_PDL)) == len(dw.bufs)
     assert aio.aio_decode_step_check(dw.step_handle(M)) == 0
     check_workload(dw, M, f"{name} M={M}")
     dw.close()
 
 
-@pytest.mark.parametrize("flags", [0, 1, 2, 3])
+@pytest.mark.parametrize("flags", [0, 1, 2, 3, 4, 5, 7])
 def test_step_flag_variants_agree(aio, flags):
     from paper_2604_09752_gb300.workload import DeviceWorkload
     dw = DeviceWorkload(swl.WORKLOADS["1b-bf16"], seed=2, max_M=2, projs=small_decoder("1b-bf16", 1))
@@ -99,18 +100,19 @@ def test_step_reads_x_only_after_previous_projection(aio):
     YA = torch.empty(NA, dtype=torch.float32, device="cuda")
     YB = torch.empty(NB, dtype=torch.float32, device="cuda")
     torch.cuda.synchronize()
-    step = aio.aio_decode_step_create([(ha, XA.data_ptr(), WA.data_ptr(), None, YA.data_ptr()),
-                                       (hb, YA.data_ptr(), WB.data_ptr(), None, YB.data_ptr())], 1)
     y_ref, mag = parity.reference(xb, wb)
-    for it in range(5):
-        YA.view(torch.int32).fill_(0x7F7F7F7F)   # garbage: huge finite bf16 halves
-        YB.zero_()
-        aio.aio_decode_step(step, torch.cuda.current_stream().cuda_stream)
-        torch.cuda.synchronize()
-        assert np.array_equal(YA.cpu().numpy(), ya[0]), "projection A wrong"
-        parity.check(YB.cpu().numpy().reshape(1, NB), y_ref, mag, KB, f"dependent projection, iteration {it}")
-    assert aio.aio_decode_step_check(step) == 0
-    aio.aio_decode_step_destroy(step)
+    for flags in (aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT, aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL):
+        step = aio.aio_decode_step_create([(ha, XA.data_ptr(), WA.data_ptr(), None, YA.data_ptr()),
+                                           (hb, YA.data_ptr(), WB.data_ptr(), None, YB.data_ptr())], 1, flags)
+        for it in range(5):
+            YA.view(torch.int32).fill_(0x7F7F7F7F)   # garbage: huge finite bf16 halves
+            YB.zero_()
+            aio.aio_decode_step(step, torch.cuda.current_stream().cuda_stream)
+            torch.cuda.synchronize()
+            assert np.array_equal(YA.cpu().numpy(), ya[0]), "projection A wrong"
+            parity.check(YB.cpu().numpy().reshape(1, NB), y_ref, mag, KB, f"flags={flags} iteration {it}")
+        assert aio.aio_decode_step_check(step) == 0
+        aio.aio_decode_step_destroy(step)
     aio.aio_linear_destroy(ha)
     aio.aio_linear_destroy(hb)
 
