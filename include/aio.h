@@ -155,6 +155,35 @@ aio_status aio_linear_unpack(aio_linear_t h, const void* W_packed, void* W_rowma
 aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, const void* W,
                           const void* scales, float* y, void* stream);
 
+/*
+ * y = x W^T as aio_linear_run computes it, without a handle and without allocating anything.
+ * The paper has no counterpart: this is a library entry for callers that cannot allocate device
+ * memory where they call -- a serving engine that has handed nearly all of HBM to its own pools
+ * (weights, KV cache), so that a cudaMalloc there fails, or a hot loop in which cudaMalloc /
+ * cudaFree would synchronise the device.
+ *   x, M, W, scales, y   as for aio_linear_run, with 1 <= M <= 8
+ *   K, N          as for aio_linear_create
+ *   wt            AIO_W_BF16 or AIO_W_INT8_PERCHANNEL
+ *   flags         AIO_FLAG_ROWMAJOR and / or AIO_FLAG_NO_PDL
+ *   device_error  device int, 4-byte aligned, owned by the caller: set non-zero if a bounded
+ *                 device-side wait expired (y is then incomplete); the library never clears it
+ * Scratch: the cross-warp partial sums and tile counters live in one static device array of
+ * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs
+ * 512 M S bytes of partial sums (S = the device's SM count) plus 4 ceil(N / 8) bytes of counters,
+ * each rounded up to 256
+ * (on a 152-SM GB300 at M = 8: N up to 851968); a larger call returns AIO_ERR_INVALID_ARG and
+ * launches nothing.  Each call enqueues a cudaMemsetAsync that zeroes the counters, then the kernel.
+ * Every call on a device shares that scratch: calls that overlap in time race and give wrong
+ * results, so issue them on one stream or order their streams.
+ * The first call on each device looks up the scratch address (cudaGetSymbolAddress) and sets the
+ * kernels' attributes; make that first call before any stream capture begins.
+ * Errors: INVALID_ARG, ALIGNMENT, UNSUPPORTED, CUDA.
+ */
+#define AIO_NOALLOC_SCRATCH_BYTES 1048576
+aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N, aio_wtype wt, unsigned flags,
+                                  const void* W, const void* scales, float* y, int* device_error,
+                                  void* stream);
+
 /* Synchronise the device, then report the handle's device error word:
  * AIO_OK, or AIO_ERR_DEVICE_TIMEOUT (code also stored in *device_error if non-NULL). */
 aio_status aio_linear_check(aio_linear_t h, int* device_error);

@@ -41,6 +41,7 @@ AIO_STEP_PDL = 0x2
 AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 8
 AIO_K_TILE = 256
+AIO_NOALLOC_SCRATCH_BYTES = 1048576
 for _name, _val in re.findall(r"#define\s+(AIO_\w+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", _hdr):
     if _name in globals() and globals()[_name] != int(_val, 0):
         raise ImportError(f"binding constant {_name} disagrees with include/aio.h")
@@ -72,6 +73,7 @@ _SIGS = {
     "aio_linear_pack": (_int, [_vp, _vp, _vp, _vp, _vp, _vp]),
     "aio_linear_unpack": (_int, [_vp, _vp, _vp, _vp]),
     "aio_linear_run": (_int, [_vp, _vp, _int, _int, _int, _vp, _vp, _vp, _vp]),
+    "aio_linear_run_noalloc": (_int, [_vp, _int, _int, _int, _int, _u, _vp, _vp, _vp, _vp, _vp]),
     "aio_linear_check": (_int, [_vp, ctypes.POINTER(_int)]),
     "aio_linear_reset": (_int, [_vp]),
     "aio_linear_destroy": (_int, [_vp]),
@@ -139,6 +141,12 @@ def aio_linear_unpack(h: int, W_packed: int, W_rowmajor: int, stream: int = 0):
 
 def aio_linear_run(h: int, x: int, M: int, K: int, N: int, W: int, scales, y: int, stream: int = 0):
     _check(_lib.aio_linear_run(h, x, M, K, N, W, scales, y, stream), "aio_linear_run")
+
+
+def aio_linear_run_noalloc(x: int, M: int, K: int, N: int, wt: int, flags: int, W: int, scales, y: int,
+                           device_error: int, stream: int = 0):
+    _check(_lib.aio_linear_run_noalloc(x, M, K, N, wt, flags, W, scales, y, device_error, stream),
+           "aio_linear_run_noalloc")
 
 
 def aio_linear_check(h: int) -> int:

@@ -579,3 +579,100 @@ aio_status aio_probe_read(const void* buf, size_t bytes, unsigned* out, void* st
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------------
+// aio_linear_run_noalloc: the single-projection launch of aio_linear_run with its cross-warp
+// scratch (partial sums of row groups split between warps, and their tile counters) in one static
+// device array that is part of the library image, instead of a handle's cudaMalloc'd workspace.
+// It is for callers that cannot allocate device memory where they call: a serving engine that has
+// handed nearly all of HBM to its own pools (weights, KV cache), so that a cudaMalloc there fails,
+// or a hot loop in which cudaMalloc / cudaFree would synchronise the device.
+
+static __device__ __align__(256) unsigned char aio_noalloc_scratch[AIO_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_base[64] = {};   // device address of aio_noalloc_scratch, per device ordinal
+
+// Looked up once per device, with that device current (the caller made it current).
+aio_status noalloc_scratch(int dev, void** out) {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_base[dev]) {
+        void* p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, aio_noalloc_scratch);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(AIO_ERR_CUDA, "cudaGetSymbolAddress(scratch) on device %d: %s", dev, cudaGetErrorString(e));
+        }
+        if (!p || !aligned(p, 256)) return fail(AIO_ERR_CUDA, "static scratch on device %d is not 256-byte aligned", dev);
+        g_noalloc_base[dev] = p;
+    }
+    *out = g_noalloc_base[dev];
+    return AIO_OK;
+}
+
+}  // namespace
+
+extern "C" aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N, aio_wtype wt, unsigned flags,
+                                             const void* W, const void* scales, float* y, int* device_error,
+                                             void* stream) {
+    if (K < 16 || K > (1 << 20) || K % 16 != 0) return fail(AIO_ERR_INVALID_ARG, "K=%d: need 16 <= K <= 2^20, K %% 16 == 0", K);
+    if (N < 1 || N > (1 << 24)) return fail(AIO_ERR_INVALID_ARG, "N=%d: need 1 <= N <= 2^24", N);
+    if (wt != AIO_W_BF16 && wt != AIO_W_INT8_PERCHANNEL) return fail(AIO_ERR_INVALID_ARG, "unknown weight type %d", (int)wt);
+    if (M < 1 || M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, 8]", M);
+    const unsigned allowed = AIO_FLAG_ROWMAJOR | AIO_FLAG_NO_PDL;
+    if (flags & ~allowed) return fail(AIO_ERR_INVALID_ARG, "unknown flags 0x%x (ROWMAJOR and NO_PDL only)", flags & ~allowed);
+    if (!x || !W || !y || !device_error) return fail(AIO_ERR_INVALID_ARG, "x, W, y and device_error must be non-NULL");
+    if (!aligned(x, 16) || !aligned(W, 16) || !aligned(y, 16))
+        return fail(AIO_ERR_ALIGNMENT, "x, W and y must be 16-byte aligned");
+    if (!aligned(device_error, 4)) return fail(AIO_ERR_ALIGNMENT, "device_error must be 4-byte aligned");
+    if (wt == AIO_W_INT8_PERCHANNEL) {
+        if (!scales) return fail(AIO_ERR_INVALID_ARG, "int8 weights need per-channel scales");
+        if (!aligned(scales, 2)) return fail(AIO_ERR_ALIGNMENT, "scales must be 2-byte aligned");
+    } else if (scales) {
+        return fail(AIO_ERR_INVALID_ARG, "bf16 weights take no scales (pass NULL)");
+    }
+    int dev = 0, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    const aio::Geometry geo = aio::geometry(K, N, sms);
+    const size_t need = aio::workspace_bytes(geo, M);
+    if (need > AIO_NOALLOC_SCRATCH_BYTES)
+        return fail(AIO_ERR_INVALID_ARG,
+                    "K=%d N=%d M=%d needs %zu bytes of scratch; the static scratch holds %zu "
+                    "(use aio_linear_create + aio_linear_run)", K, N, M, need, (size_t)AIO_NOALLOC_SCRATCH_BYTES);
+    void* base = nullptr;
+    if ((st = noalloc_scratch(dev, &base)) != AIO_OK) return st;
+    float* partial = nullptr;
+    unsigned* counters = nullptr;
+    aio::carve_workspace(base, geo, M, &partial, &counters);
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // The tile counters must start at zero; a healthy run leaves them zero, an expired wait may not.
+    AIO_CUDA(cudaMemsetAsync(counters, 0, static_cast<size_t>(geo.NG) * sizeof(unsigned), s));
+    aio::ProjDesc d = {};
+    d.x = static_cast<const uint16_t*>(x);
+    d.w = static_cast<const uint8_t*>(W);
+    d.scales = static_cast<const uint16_t*>(scales);
+    d.y = y;
+    d.partial = partial;
+    d.counters = counters;
+    d.T = geo.T;
+    d.K = K;
+    d.N = N;
+    d.NG = geo.NG;
+    d.NKT = geo.NKT;
+    d.rowmajor = (flags & AIO_FLAG_ROWMAJOR) ? 1 : 0;
+    d.uniform = (!d.rowmajor && N % aio::kRows == 0 && K % aio::kKT == 0) ? 1 : 0;
+    aio::StreamArgs a = {};
+    a.projs = nullptr;
+    a.one = d;
+    a.err = device_error;
+    a.nproj = 1;
+    a.M = M;
+    a.Z = geo.Z;
+    a.test_stall = 0;
+    a.wait_limit_ns = kWaitLimitNs;
+    AIO_CUDA(aio::launch_stream(a, wt == AIO_W_INT8_PERCHANNEL, geo.grid, s, !(flags & AIO_FLAG_NO_PDL), false));
+    return AIO_OK;
+}
