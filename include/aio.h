@@ -114,7 +114,7 @@ const char* aio_last_error(void);
  *   wt     AIO_W_BF16 or AIO_W_INT8_PERCHANNEL
  *   max_M  1..8: the largest number of token rows later passed to aio_linear_run
  *   flags  AIO_FLAG_* bits
- * Allocates a small device workspace (cross-CTA partial sums and counters, zeroed here)
+ * Allocates a small device workspace (cross-warp partial sums and an error word, set up here)
  * on the current device; synchronises that device.  Errors: INVALID_ARG, UNSUPPORTED,
  * OOM, CUDA.
  */
@@ -167,12 +167,12 @@ aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, co
  *   flags         AIO_FLAG_ROWMAJOR and / or AIO_FLAG_NO_PDL
  *   device_error  device int, 4-byte aligned, owned by the caller: set non-zero if a bounded
  *                 device-side wait expired (y is then incomplete); the library never clears it
- * Scratch: the cross-warp partial sums and tile counters live in one static device array of
- * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs
- * 512 M S bytes of partial sums (S = the device's SM count) plus 4 ceil(N / 8) bytes of counters,
- * each rounded up to 256
- * (on a 152-SM GB300 at M = 8: N up to 851968); a larger call returns AIO_ERR_INVALID_ARG and
- * launches nothing.  Each call enqueues a cudaMemsetAsync that zeroes the counters, then the kernel.
+ * Scratch: the cross-warp partial sums live in one static device array of
+ * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs 256 M S
+ * bytes of it (S = the device's SM count), rounded up to 256: on a 152-SM GB300 every M <= 8 fits
+ * (311296 bytes at M = 8).  A call that needs more returns AIO_ERR_INVALID_ARG and launches nothing.
+ * Each call enqueues a cudaMemsetAsync that empties the partial-sum slots it uses (all bytes 0xFF),
+ * then the kernel.
  * Every call on a device shares that scratch: calls that overlap in time race and give wrong
  * results, so issue them on one stream or order their streams.
  * The first call on each device looks up the scratch address (cudaGetSymbolAddress) and sets the
@@ -188,7 +188,7 @@ aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N, aio_wtype 
  * AIO_OK, or AIO_ERR_DEVICE_TIMEOUT (code also stored in *device_error if non-NULL). */
 aio_status aio_linear_check(aio_linear_t h, int* device_error);
 
-/* Clear the handle's workspace counters and error word (needed only after a device error). */
+/* Empty the handle's partial-sum slots and clear its error word (needed only after a device error). */
 aio_status aio_linear_reset(aio_linear_t h);
 
 /* Free the handle and its workspace (synchronises the device). NULL is accepted. */
@@ -211,7 +211,7 @@ aio_status aio_decode_step(aio_step_t step, void* stream);
 /* Number of kernels one aio_decode_step launches (1 in persistent mode, else one per projection). */
 aio_status aio_decode_step_kernels(aio_step_t step, int* n_kernels);
 
-/* Clear the step's workspace counters and error words (needed only after a device error). */
+/* Empty the step's partial-sum slots, clear its counters and error words (needed only after a device error). */
 aio_status aio_decode_step_reset(aio_step_t step);
 
 /* Synchronise the device, then report the step's device error word (see aio_linear_check). */

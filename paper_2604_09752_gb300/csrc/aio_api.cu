@@ -2,6 +2,8 @@
 // workspaces, kernel launches, and the decode step captured as one CUDA graph.
 #include <cuda_runtime.h>
 
+#include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
@@ -70,6 +72,133 @@ aio_status current_device(int* dev, int* sms) {
     return AIO_OK;
 }
 
+// ---------------------------------------------------------------------------------------------
+// Balanced partition.  Under full load the SMs of a GB300 do not stream at one rate: for equal
+// shares some finish up to a third later than others, the same SMs every time (the spread follows
+// the chip's layout, not the data).  In a decode step every projection ends at a grid-wide
+// barrier, so equal shares leave the fast SMs idle at every barrier.  Once per device we measure
+// how long each CTA of a full-grid read takes and move the CTAs' shares toward equal finish times
+// (a few rounds, each rescaling a CTA's weight by mean time / its time).  The table is fixed for
+// the life of the process, so results stay deterministic run to run.  Shares are keyed by CTA
+// index, so the partition is correct whatever SM a CTA lands on; only its balance depends on it.
+// AIO_BALANCE=0 in the environment keeps equal shares.
+std::mutex g_bal_mu;
+bool g_bal_done[64] = {};
+const unsigned* g_bal_cw[64] = {};
+float g_bal_spread[64][2] = {};       // max/min CTA time for equal shares, and for the final table
+
+void cw_from_weights(const std::vector<double>& w, int warps, std::vector<unsigned>& cw) {
+    const int Z = static_cast<int>(w.size()) * warps;
+    double total = 0;
+    for (double v : w) total += v;
+    cw.assign(Z + 1, 0u);
+    double acc = 0;
+    for (int z = 0; z < Z; ++z) {
+        cw[z] = static_cast<unsigned>(std::llround(acc / total * static_cast<double>(1u << aio::kCwShift)));
+        acc += w[z / warps] / warps;
+    }
+    cw[Z] = 1u << aio::kCwShift;
+    for (int z = 1; z <= Z; ++z) cw[z] = std::max(cw[z], cw[z - 1]);
+}
+
+// Per-CTA time of one full-grid read of `bytes` under table cw (null: equal shares), in seconds.
+bool probe_cta_times(const void* buf, size_t bytes, int sms, const unsigned* cw, unsigned* out,
+                     unsigned long long* rec, std::vector<unsigned long long>& h, std::vector<double>& t) {
+    const int Z = sms * aio::kWarps;
+    for (int rep = 0; rep < 2; ++rep)
+        if (aio::launch_probe(buf, static_cast<long long>(bytes / 4096), out, sms, nullptr, cw, rec) != cudaSuccess)
+            return false;
+    if (cudaDeviceSynchronize() != cudaSuccess) return false;
+    h.resize(2 * static_cast<size_t>(Z));
+    if (cudaMemcpy(h.data(), rec, h.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return false;
+    unsigned long long t0 = ~0ull;
+    for (int z = 0; z < Z; ++z) {
+        if (h[2 * z] == 0 || h[2 * z + 1] < h[2 * z]) return false;
+        t0 = std::min(t0, h[2 * z]);
+    }
+    t.assign(sms, 0.0);
+    for (int z = 0; z < Z; ++z)
+        t[z / aio::kWarps] = std::max(t[z / aio::kWarps], static_cast<double>(h[2 * z + 1] - t0) * 1e-9);
+    return true;
+}
+
+// Builds (once) the calibrated table of the current device `dev`; leaves null (equal shares) when
+// disabled or when the measurement cannot be made.  Synchronises the device.
+void balance_table(int dev, int sms, const unsigned** out) {
+    std::lock_guard<std::mutex> lk(g_bal_mu);
+    if (g_bal_done[dev]) {
+        *out = g_bal_cw[dev];
+        return;
+    }
+    g_bal_done[dev] = true;
+    *out = nullptr;
+    const char* env = getenv("AIO_BALANCE");
+    if (env && env[0] == '0') return;
+    const int Z = sms * aio::kWarps;
+    const size_t cw_bytes = round_up(sizeof(unsigned) * (Z + 1), 256);
+    unsigned* table = nullptr;
+    if (cudaMalloc(&table, cw_bytes) != cudaSuccess) {
+        cudaGetLastError();
+        return;
+    }
+    void* scratch = nullptr;
+    const size_t rec_bytes = round_up(sizeof(unsigned long long) * 2 * Z, 256);
+    size_t bytes = size_t(1) << 30;
+    while (bytes >= (size_t(256) << 20) && cudaMalloc(&scratch, bytes + rec_bytes + 256) != cudaSuccess) {
+        cudaGetLastError();
+        scratch = nullptr;
+        bytes /= 2;
+    }
+    if (!scratch) {
+        cudaFree(table);
+        return;
+    }
+    uint8_t* base = static_cast<uint8_t*>(scratch);
+    auto* rec = reinterpret_cast<unsigned long long*>(base + bytes);
+    auto* xo = reinterpret_cast<unsigned*>(base + bytes + rec_bytes);
+    std::vector<unsigned long long> h;
+    std::vector<double> t, w(sms, 1.0), best_w;
+    std::vector<unsigned> cw;
+    double best = 1e30;
+    bool ok = probe_cta_times(base, bytes, sms, nullptr, xo, rec, h, t);   // warm-up and equal shares
+    if (ok) ok = probe_cta_times(base, bytes, sms, nullptr, xo, rec, h, t);
+    if (ok) {
+        const auto mm = std::minmax_element(t.begin(), t.end());
+        g_bal_spread[dev][0] = static_cast<float>(*mm.second / *mm.first);
+    }
+    for (int it = 0; ok && it < 5; ++it) {
+        double mean = 0;
+        for (double v : t) mean += v / sms;
+        for (int b = 0; b < sms; ++b) w[b] = std::min(2.0, std::max(0.5, w[b] * mean / t[b]));
+        cw_from_weights(w, aio::kWarps, cw);
+        ok = cudaMemcpy(table, cw.data(), sizeof(unsigned) * (Z + 1), cudaMemcpyHostToDevice) == cudaSuccess &&
+             probe_cta_times(base, bytes, sms, table, xo, rec, h, t);
+        if (!ok) break;
+        const auto mm = std::minmax_element(t.begin(), t.end());
+        if (*mm.second < best) {
+            best = *mm.second;
+            best_w = w;
+            g_bal_spread[dev][1] = static_cast<float>(*mm.second / *mm.first);
+        }
+    }
+    if (ok && !best_w.empty()) {
+        cw_from_weights(best_w, aio::kWarps, cw);
+        ok = cudaMemcpy(table, cw.data(), sizeof(unsigned) * (Z + 1), cudaMemcpyHostToDevice) == cudaSuccess;
+    }
+    cudaFree(scratch);
+    if (!ok || best_w.empty()) {
+        cudaGetLastError();
+        cudaFree(table);
+        return;
+    }
+    g_bal_cw[dev] = table;
+    *out = table;
+    if (getenv("AIO_BALANCE_LOG"))
+        fprintf(stderr, "libaio: device %d balance: CTA time spread %.3f with equal shares, %.3f calibrated\n", dev,
+                g_bal_spread[dev][0], g_bal_spread[dev][1]);
+}
+
 aio_status check_device(int dev) {
     int cur = -1;
     AIO_CUDA(cudaGetDevice(&cur));
@@ -92,15 +221,7 @@ Geometry geometry(int K, int N, int num_sms) {
 }
 
 size_t workspace_bytes(const Geometry& g, int M) {
-    return round_up(static_cast<size_t>(g.Z) * 2 * kRows * M * sizeof(float), 256) +
-           round_up(static_cast<size_t>(g.NG) * sizeof(unsigned), 256);
-}
-
-void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters) {
-    uint8_t* p = static_cast<uint8_t*>(base);
-    *partial = reinterpret_cast<float*>(p);
-    p += round_up(static_cast<size_t>(g.Z) * 2 * kRows * M * sizeof(float), 256);
-    *counters = reinterpret_cast<unsigned*>(p);
+    return round_up(static_cast<size_t>(g.Z) * kRows * M * sizeof(float), 256);
 }
 
 }  // namespace aio
@@ -112,11 +233,11 @@ struct aio_linear {
     unsigned flags;
     int device;
     aio::Geometry geo;
-    void* ws;            // partial sums, counters, then the error word
+    void* ws;            // partial-sum slots, then the error word
     size_t ws_bytes;
-    float* partial;
-    unsigned* counters;
+    float* partial;      // partial-sum slots (empty pattern 0xFF at rest)
     int* err;
+    const unsigned* cw;  // the device's balanced partition table (null: equal shares)
 };
 
 struct aio_step {
@@ -145,14 +266,13 @@ aio_status valid_linear(aio_linear_t h) {
 }
 
 aio::ProjDesc make_desc(const aio_linear* h, const void* x, const void* W, const void* scales, float* y,
-                        float* partial, unsigned* counters) {
+                        float* partial) {
     aio::ProjDesc d = {};
     d.x = static_cast<const uint16_t*>(x);
     d.w = static_cast<const uint8_t*>(W);
     d.scales = static_cast<const uint16_t*>(scales);
     d.y = y;
     d.partial = partial;
-    d.counters = counters;
     d.T = h->geo.T;
     d.K = h->K;
     d.N = h->N;
@@ -173,6 +293,7 @@ aio::StreamArgs single_args(const aio_linear* h, const aio::ProjDesc& d, int M, 
     a.nproj = 1;
     a.M = M;
     a.Z = h->geo.Z;
+    a.cw = h->cw;
     a.test_stall = (h->flags & AIO_FLAG_TEST_STALL) ? 1 : 0;
     a.wait_limit_ns = a.test_stall ? kTestWaitLimitNs : kWaitLimitNs;
     return a;
@@ -227,13 +348,16 @@ aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int 
     if (st != AIO_OK) return st;
     aio::Geometry geo = aio::geometry(K, N, sms);
     const size_t ws = aio::workspace_bytes(geo, max_M);
+    const unsigned* cw = nullptr;
+    balance_table(dev, sms, &cw);
     if (test_alloc_failure()) return fail(AIO_ERR_OOM, "workspace allocation failed (AIO_TEST_FAIL_ALLOC)");
     void* mem = nullptr;
     if (cudaMalloc(&mem, ws + 256) != cudaSuccess) {
         cudaGetLastError();
         return fail(AIO_ERR_OOM, "cudaMalloc(%zu) failed", ws + 256);
     }
-    if (cudaMemset(mem, 0, ws + 256) != cudaSuccess || cudaDeviceSynchronize() != cudaSuccess) {
+    if (cudaMemset(mem, 0xFF, ws) != cudaSuccess || cudaMemset(static_cast<uint8_t*>(mem) + ws, 0, 256) != cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess) {
         cudaFree(mem);
         return fail(AIO_ERR_CUDA, "workspace initialisation failed");
     }
@@ -252,8 +376,9 @@ aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int 
     h->geo = geo;
     h->ws = mem;
     h->ws_bytes = ws + 256;
-    aio::carve_workspace(mem, geo, max_M, &h->partial, &h->counters);
+    h->partial = static_cast<float*>(mem);
     h->err = reinterpret_cast<int*>(static_cast<uint8_t*>(mem) + ws);
+    h->cw = cw;
     *out = h;
     return AIO_OK;
 }
@@ -319,7 +444,7 @@ aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, co
     if (K != h->K || N != h->N) return fail(AIO_ERR_INVALID_ARG, "K=%d N=%d do not match the handle (K=%d N=%d)", K, N, h->K, h->N);
     if ((st = validate_run(h, x, M, W, scales, y)) != AIO_OK) return st;
     if ((st = check_device(h->device)) != AIO_OK) return st;
-    const aio::StreamArgs a = single_args(h, make_desc(h, x, W, scales, y, h->partial, h->counters), M, h->err);
+    const aio::StreamArgs a = single_args(h, make_desc(h, x, W, scales, y, h->partial), M, h->err);
     AIO_CUDA(aio::launch_stream(a, h->wt == AIO_W_INT8_PERCHANNEL, h->geo.grid, static_cast<cudaStream_t>(stream),
                                 !(h->flags & AIO_FLAG_NO_PDL), false));
     return AIO_OK;
@@ -349,7 +474,8 @@ aio_status aio_linear_reset(aio_linear_t h) {
     if (st != AIO_OK) return st;
     if ((st = check_device(h->device)) != AIO_OK) return st;
     AIO_CUDA(cudaDeviceSynchronize());
-    AIO_CUDA(cudaMemset(h->ws, 0, h->ws_bytes));
+    AIO_CUDA(cudaMemset(h->ws, 0xFF, h->ws_bytes - 256));   // partial slots: empty
+    AIO_CUDA(cudaMemset(h->err, 0, 256));
     AIO_CUDA(cudaDeviceSynchronize());
     return AIO_OK;
 }
@@ -455,10 +581,7 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     std::vector<aio::ProjDesc> descs;
     for (int i = 0; i < n_projs; ++i) {
         const aio_proj& p = projs[i];
-        float* partial = nullptr;
-        unsigned* counters = nullptr;
-        aio::carve_workspace(base + offs[i], p.h->geo, M, &partial, &counters);
-        descs.push_back(make_desc(p.h, p.x, p.W, p.scales, p.y, partial, counters));
+        descs.push_back(make_desc(p.h, p.x, p.W, p.scales, p.y, reinterpret_cast<float*>(base + offs[i])));
         s->chain.push_back(single_args(p.h, descs.back(), M, s->errs + i));
         s->chain_i8.push_back(p.h->wt == AIO_W_INT8_PERCHANNEL ? 1 : 0);
     }
@@ -470,10 +593,12 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     w.nproj = n_projs;
     w.M = M;
     w.Z = projs[0].h->geo.Z;
+    w.cw = projs[0].h->cw;
     w.test_stall = 0;
     w.wait_limit_ns = kWaitLimitNs;
     s->whole = w;
-    if (cudaMemset(s->ws, 0, total) != cudaSuccess ||
+    if (cudaMemset(s->ws, 0xFF, desc_off) != cudaSuccess ||
+        cudaMemset(base + desc_off, 0, total - desc_off) != cudaSuccess ||
         cudaMemcpy(base + desc_off, descs.data(), sizeof(aio::ProjDesc) * n_projs, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess) {
         step_free(s);
@@ -541,7 +666,7 @@ aio_status aio_decode_step_reset(aio_step_t s) {
     const size_t desc_off = reinterpret_cast<const uint8_t*>(s->whole.projs) - static_cast<const uint8_t*>(s->ws);
     const size_t done_off = reinterpret_cast<const uint8_t*>(s->whole.done) - static_cast<const uint8_t*>(s->ws);
     AIO_CUDA(cudaDeviceSynchronize());
-    AIO_CUDA(cudaMemset(s->ws, 0, desc_off));   // partial sums and tile counters
+    AIO_CUDA(cudaMemset(s->ws, 0xFF, desc_off));   // partial-sum slots: empty
     AIO_CUDA(cudaMemset(static_cast<uint8_t*>(s->ws) + done_off, 0, s->ws_bytes - done_off));  // done, errors
     AIO_CUDA(cudaDeviceSynchronize());
     return AIO_OK;
@@ -582,7 +707,7 @@ aio_status aio_probe_read(const void* buf, size_t bytes, unsigned* out, void* st
 
 // ---------------------------------------------------------------------------------------------
 // aio_linear_run_noalloc: the single-projection launch of aio_linear_run with its cross-warp
-// scratch (partial sums of row groups split between warps, and their tile counters) in one static
+// scratch (partial sums of row groups split between warps) in one static
 // device array that is part of the library image, instead of a handle's cudaMalloc'd workspace.
 // It is for callers that cannot allocate device memory where they call: a serving engine that has
 // handed nearly all of HBM to its own pools (weights, KV cache), so that a cudaMalloc there fails,
@@ -638,25 +763,26 @@ extern "C" aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N,
     if (st != AIO_OK) return st;
     const aio::Geometry geo = aio::geometry(K, N, sms);
     const size_t need = aio::workspace_bytes(geo, M);
-    if (need > AIO_NOALLOC_SCRATCH_BYTES)
+    size_t limit = AIO_NOALLOC_SCRATCH_BYTES;
+    if (const char* t = getenv("AIO_TEST_NOALLOC_BYTES"))   // test hook: a smaller limit
+        limit = std::min(limit, static_cast<size_t>(strtoull(t, nullptr, 10)));
+    if (need > limit)
         return fail(AIO_ERR_INVALID_ARG,
                     "K=%d N=%d M=%d needs %zu bytes of scratch; the static scratch holds %zu "
-                    "(use aio_linear_create + aio_linear_run)", K, N, M, need, (size_t)AIO_NOALLOC_SCRATCH_BYTES);
+                    "(use aio_linear_create + aio_linear_run)", K, N, M, need, limit);
     void* base = nullptr;
     if ((st = noalloc_scratch(dev, &base)) != AIO_OK) return st;
-    float* partial = nullptr;
-    unsigned* counters = nullptr;
-    aio::carve_workspace(base, geo, M, &partial, &counters);
+    float* partial = static_cast<float*>(base);
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // The tile counters must start at zero; a healthy run leaves them zero, an expired wait may not.
-    AIO_CUDA(cudaMemsetAsync(counters, 0, static_cast<size_t>(geo.NG) * sizeof(unsigned), s));
+    // The partial-sum slots must start empty (all bytes 0xFF); a healthy run leaves them so, an
+    // expired wait may not, and the array starts out zeroed.
+    AIO_CUDA(cudaMemsetAsync(partial, 0xFF, need, s));
     aio::ProjDesc d = {};
     d.x = static_cast<const uint16_t*>(x);
     d.w = static_cast<const uint8_t*>(W);
     d.scales = static_cast<const uint16_t*>(scales);
     d.y = y;
     d.partial = partial;
-    d.counters = counters;
     d.T = geo.T;
     d.K = K;
     d.N = N;

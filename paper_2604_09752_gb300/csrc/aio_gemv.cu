@@ -26,9 +26,12 @@
 //     operations and one bf16x2 subtraction per pair; the per-channel scale multiplies the
 //     finished fp32 sum.
 //   * Split row groups.  A row group whose tiles all lie in one warp's segment is written directly.
-//     One split between warps is finished by the last warp to add its tile count to the group's
-//     counter: contributors store partial sums, fence, count; the last one sums the partials in
-//     warp order (deterministic), writes y and resets the counter.  Nothing spins.
+//     A group split between warps is owned by its first contributor, for which it is the last group
+//     of its segment, so the owner reaches it at the end of the phase; the other contributors reach
+//     it earlier, at the start of their segments.  They store their partial sums with relaxed
+//     stores into slots that read 0xFFFFFFFF (a bit pattern no computed float takes) while empty,
+//     and move on: no fence and no atomic on their path.  The owner polls the slots (bounded),
+//     sums them in warp order (deterministic), writes y and empties the slots again.
 //   * Projection order.  In a persistent step, projection p+1 reads x only after every CTA has
 //     finished projection p: warps count in shared memory, the last warp of a CTA makes one global
 //     increment, warp 0 of each CTA polls the global counter (bounded) and publishes it to its CTA.
@@ -100,6 +103,29 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;"
         ::"r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
         : "memory");
+}
+
+// The same without an L2 cache hint (activations: read by every CTA, keep the default policy).
+__device__ __forceinline__ void bulk_g2s_plain(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ void st_relaxed_u32(void* p, uint32_t v) {
+    asm volatile("st.relaxed.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_relaxed_u32(const void* p) {
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
 
 __device__ __forceinline__ void fence_proxy_async_smem() {
@@ -230,6 +256,12 @@ __device__ __forceinline__ void issue_chunk(const ProjDesc* d, int t, int nt, ui
 }
 
 // A warp's walk over its tiles of every projection, one chunk (<= C consecutive tiles) at a time.
+// First tile of warp z's segment of a projection with T tiles (z = Z gives T).
+__device__ __forceinline__ long long seg_start(const unsigned* cw, long long z, int Z, long long T) {
+    if (cw) return (T * static_cast<long long>(__ldg(cw + z))) >> kCwShift;
+    return z * T / Z;
+}
+
 struct ChunkCursor {
     int p, t, te;
 };
@@ -237,8 +269,8 @@ struct ChunkCursor {
 __device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, long long z, int Z) {
     const long long T = proj_desc(s, 0)->T;
     c.p = 0;
-    c.t = static_cast<int>(z * T / Z);
-    c.te = static_cast<int>((z + 1) * T / Z);
+    c.t = static_cast<int>(seg_start(s.cw, z, Z, T));
+    c.te = static_cast<int>(seg_start(s.cw, z + 1, Z, T));
 }
 
 // Next chunk of the walk: its projection, first tile and tile count; false at the end.
@@ -248,8 +280,8 @@ __device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s,
         if (c.p + 1 >= s.nproj) return false;
         ++c.p;
         const long long T = proj_desc(s, c.p)->T;
-        c.t = static_cast<int>(z * T / Z);
-        c.te = static_cast<int>((z + 1) * T / Z);
+        c.t = static_cast<int>(seg_start(s.cw, z, Z, T));
+        c.te = static_cast<int>(seg_start(s.cw, z + 1, Z, T));
     }
     p = c.p;
     t = c.t;
@@ -264,7 +296,6 @@ struct Proj {
     const uint16_t* scales;
     float* y;
     float* partial;
-    unsigned* counters;
     long long T;
     int M, K, N, NKT;
     int rowmajor, uniform;
@@ -276,7 +307,6 @@ __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
     p.scales = d->scales;
     p.y = d->y;
     p.partial = d->partial;
-    p.counters = d->counters;
     p.T = d->T;
     p.M = M;
     p.K = d->K;
@@ -380,6 +410,40 @@ __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* t
     }
 }
 
+// The same with x staged in shared memory: xaddr is the shared-window address of this lane's
+// x piece 0 for the tile (token min(g, M-1), k = 256 kt + 64c); W and x both come in with
+// ld.shared.v4.  Lanes with g >= M load a real token's x: they fill rows of A whose outputs
+// (tokens >= M) are never written, so no select is needed.
+template <bool I8>
+__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr) {
+    using TL = TileT<I8>;
+    constexpr int NP = TL::kPieces;
+    uint4 w[NP];
+#pragma unroll
+    for (int j = 0; j < NP; ++j) w[j] = lds128(waddr + j * 512);
+    uint4 xv[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) xv[j] = lds128(xaddr + 16 * j);
+#pragma unroll
+    for (int s = 0; s < 16; ++s) {
+        const uint4& xq = xv[s >> 1];
+        const uint32_t a0 = (s & 1) ? xq.z : xq.x;
+        const uint32_t a2 = (s & 1) ? xq.w : xq.y;
+        uint32_t b0, b1;
+        if constexpr (I8) {
+            const uint4& wq = w[s >> 2];
+            const uint32_t word = (s & 3) == 0 ? wq.x : (s & 3) == 1 ? wq.y : (s & 3) == 2 ? wq.z : wq.w;
+            b0 = i8x2_to_bf16x2<0x4140u>(word);
+            b1 = i8x2_to_bf16x2<0x4342u>(word);
+        } else {
+            const uint4& wq = w[s >> 1];
+            b0 = (s & 1) ? wq.z : wq.x;
+            b1 = (s & 1) ? wq.w : wq.y;
+        }
+        mma_bf16(d[s & 3], a0, 0u, a2, 0u, b0, b1);
+    }
+}
+
 template <bool I8>
 __device__ __forceinline__ float row_scale(const Proj& P, int n) {
     if constexpr (I8) {
@@ -389,61 +453,80 @@ __device__ __forceinline__ float row_scale(const Proj& P, int n) {
     }
 }
 
+constexpr uint32_t kSlotEmpty = 0xFFFFFFFFu;   // a partial slot not written yet
+
+// A partial sum as stored in a slot: NaNs become the quiet NaN 0x7FC00000, so no stored value is
+// ever kSlotEmpty.
+__device__ __forceinline__ uint32_t slot_bits(float v) {
+    return v != v ? 0x7FC00000u : __float_as_uint(v);
+}
+
 // Warp z has finished its tiles of row group g: lane (g', c) holds D[token g'][rows 2c, 2c+1].
-// Write y (group complete in this warp) or hand the partial to the last-arriver fixup.
+// Writes y (group complete in this warp), stores the partial (split group, not the owner), or, as
+// the owner, adds the other contributors' partials and writes y.  Returns false if a wait for a
+// partial expired or the launch already failed.
 template <bool I8>
-__device__ __forceinline__ void finish_group(const Proj& P, int Z, const float (&d)[4], int g, int rows, long long z,
-                                             long long t0, long long t1, int lane) {
+__device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s, int Z, const float (&d)[4], int g,
+                                             int rows, long long z, long long t0, long long t1, int lane) {
     const int tok = lane >> 2, r0 = 2 * (lane & 3);
     const int row0 = g * kRows;
     const long long gfirst = static_cast<long long>(g) * P.NKT;
-    const int kt_lo = t0 > gfirst ? static_cast<int>(t0 - gfirst) : 0;
-    const int kt_hi = static_cast<int>(min(static_cast<long long>(P.NKT - 1), t1 - 1 - gfirst));
+    const long long tl = gfirst + P.NKT - 1;
     const bool mine = tok < P.M;
 
-    if (kt_lo == 0 && kt_hi == P.NKT - 1) {
+    if (t0 <= gfirst && t1 > tl) {
         if (mine) {
             float* yp = P.y + static_cast<size_t>(tok) * P.N + row0 + r0;
             if (r0 < rows) yp[0] = d[0] * row_scale<I8>(P, row0 + r0);
             if (r0 + 1 < rows) yp[1] = d[1] * row_scale<I8>(P, row0 + r0 + 1);
         }
-        return;
+        return true;
     }
 
-    // Split group: publish this warp's partial [token][row], then count tiles; the warp completing
-    // the count owns the final sum.
     const int V = kRows * P.M;
-    const int side = (g == static_cast<int>(t0 / P.NKT)) ? 0 : 1;
-    float* part = P.partial + (static_cast<size_t>(z) * 2 + side) * V;
-    if (mine) {
-        part[tok * kRows + r0] = d[0];
-        part[tok * kRows + r0 + 1] = d[1];
-    }
-    __threadfence();
-    __syncwarp();
-    const unsigned ntk = static_cast<unsigned>(kt_hi - kt_lo + 1);
-    unsigned prev = 0;
-    if (lane == 0) prev = atomicAdd(&P.counters[g], ntk);
-    prev = __shfl_sync(0xffffffffu, prev, 0);
-    if (prev + ntk != static_cast<unsigned>(P.NKT)) return;
-
-    __threadfence();
-    const long long tf = gfirst, tl = gfirst + P.NKT - 1;
-    const long long zf = ((tf + 1) * Z - 1) / P.T;   // warp whose segment holds tile tf
-    const long long zl = ((tl + 1) * Z - 1) / P.T;   // ... and tile tl
-    for (int v = lane; v < V; v += 32) {
-        const int m = v / kRows, r = v - m * kRows;
-        if (r >= rows) continue;
-        float sum = 0.0f;
-        for (long long zz = zf; zz <= zl; ++zz) {
-            const long long s0 = zz * P.T / Z, s1 = (zz + 1) * P.T / Z;
-            if (s1 == s0) continue;
-            const int sd = (g == static_cast<int>(s0 / P.NKT)) ? 0 : 1;
-            sum += __ldcg(P.partial + (static_cast<size_t>(zz) * 2 + sd) * V + v);
+    if (t0 > gfirst) {
+        // Not the owner: g is this warp's first group (its last split group it always owns), so
+        // one slot per warp suffices.  Publish [token][row] and go on.
+        float* part = P.partial + static_cast<size_t>(z) * V;
+        if (mine) {
+            st_relaxed_u32(part + tok * kRows + r0, slot_bits(d[0]));
+            st_relaxed_u32(part + tok * kRows + r0 + 1, slot_bits(d[1]));
         }
-        P.y[static_cast<size_t>(m) * P.N + row0 + r] = sum * row_scale<I8>(P, row0 + r);
+        return true;
     }
-    if (lane == 0) P.counters[g] = 0u;
+
+    // The owner: this warp holds tile gfirst.  The other contributors are the next warps up to the
+    // owner of tile tl (segments are contiguous and in warp order).
+    long long zl = z;
+    while (zl + 1 < Z && seg_start(s.cw, zl + 1, Z, P.T) <= tl) ++zl;
+    bool ok = true;
+    for (int v0 = 0; v0 < V; v0 += 32) {
+        const int v = v0 + lane;
+        const int m = v / kRows, r = v - m * kRows;
+        const int src = (m * 4 + (r >> 1)) & 31;          // the lane holding the owner's own value
+        const float own0 = __shfl_sync(0xffffffffu, d[0], src);
+        const float own1 = __shfl_sync(0xffffffffu, d[1], src);
+        if (v < V && r < rows) {
+            float sum = (r & 1) ? own1 : own0;
+            for (long long zz = z + 1; ok && zz <= zl; ++zz) {
+                if (seg_start(s.cw, zz + 1, Z, P.T) == seg_start(s.cw, zz, Z, P.T)) continue;   // empty segment
+                float* slot = P.partial + static_cast<size_t>(zz) * V + v;
+                uint32_t bits = ld_relaxed_u32(slot);
+                if (bits == kSlotEmpty) {
+                    const uint64_t start = globaltimer_ns();
+                    while (ok && (bits = ld_relaxed_u32(slot)) == kSlotEmpty)
+                        ok = ld_relaxed_u32(s.err) == 0u && globaltimer_ns() - start <= s.wait_limit_ns;
+                }
+                if (ok) {
+                    sum += __uint_as_float(bits);
+                    st_relaxed_u32(slot, kSlotEmpty);
+                }
+            }
+            if (ok) P.y[static_cast<size_t>(m) * P.N + row0 + r] = sum * row_scale<I8>(P, row0 + r);
+        }
+        if (!__all_sync(0xffffffffu, ok)) return false;   // uniform: every lane reaches this point
+    }
+    return true;
 }
 
 // Lane 0 polls until *counter >= target (bounded by limit_ns); the result is broadcast to the warp.
@@ -513,6 +596,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     // CTA-level sync words: [0] warps of this CTA done with the current phase, [1] highest projection
     // index whose predecessor is known complete (published by warp 0).
     unsigned* cta_sync = reinterpret_cast<unsigned*>(smem + kSyncOffset);
+    // x of the current projection, staged once per CTA when it fits (one bulk copy by warp 0).
+    uint64_t* xbar = reinterpret_cast<uint64_t*>(smem + kSyncOffset + 16);
+    uint16_t* xs = reinterpret_cast<uint16_t*>(smem + kXsOffset);
 
     griddep_launch_dependents();
 
@@ -526,6 +612,8 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     if (threadIdx.x == 0) {
         cta_sync[0] = 0u;
         cta_sync[1] = 0u;
+        mbar_init(xbar, 1);
+        fence_mbar_init();
     }
     __syncthreads();   // the only CTA-wide barrier: barriers and sync words are initialised
     const uint64_t pol = policy_evict_first();
@@ -558,16 +646,29 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     const unsigned G = gridDim.x;
     int cslot = 0;
     uint32_t cphase = 0;
+    uint32_t xphase = 0;
     bool dead = false;    // set after a timeout: stop consuming, keep signalling
     for (int p = 0; p < s.nproj; ++p) {
-        const Proj P = load_proj(proj_desc(s, p), MT);
-        const long long t0 = z * P.T / Z, t1 = (z + 1) * P.T / Z;
+        Proj P = load_proj(proj_desc(s, p), MT);
+        const long long t0 = seg_start(s.cw, z, Z, P.T), t1 = seg_start(s.cw, z + 1, Z, P.T);
+        const uint32_t xbytes = static_cast<uint32_t>(P.M) * static_cast<uint32_t>(P.K) * 2u;
+        const bool stage = xbytes <= static_cast<uint32_t>(kXsBytes);
+        // Warp 0 stages x once every CTA has finished the previous projection (every warp of this
+        // CTA has then finished reading the previous x and fenced its reads against async writes).
+        auto stage_x = [&]() {
+            if (stage && lane == 0) {
+                mbar_expect_tx(xbar, xbytes);
+                bulk_g2s_plain(xs, P.x, xbytes, xbar);
+            }
+        };
+        if (p == 0 && warp == 0) stage_x();
         if (p > 0) {
             // Projection p reads x only after every CTA finished projection p-1.
             bool ok;
             if (warp == 0) {
                 const bool polled = !dead && poll_global(&s.done[p - 1], G, s.wait_limit_ns, lane);
                 ok = dead || polled;
+                stage_x();
                 if (lane == 0) st_release_cta_shared(&cta_sync[1], static_cast<unsigned>(p));
                 if (polled && p > 1 && blockIdx.x == 0 && lane == 0) s.done[p - 2] = 0u;   // nobody polls it any more
             } else {
@@ -579,6 +680,15 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 dead = true;
             }
         }
+        if (stage) {
+            // every warp waits for the staged x (also so that no copy is in flight at exit)
+            if (!__all_sync(0xffffffffu, mbar_wait(xbar, xphase, s.wait_limit_ns)) && !dead) {
+                if (lane == 0) atomicExch(s.err, kDevErrTimeout);
+                dead = true;
+            }
+            xphase ^= 1u;
+            P.x = xs;   // the general tile path reads the staged copy too
+        }
         if (!dead && t1 > t0) {
             float d[4][4] = {};
             const int NKT = P.NKT;
@@ -589,6 +699,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             int rows = min(kRows, P.N - g * kRows);
             const bool xrow = (lane >> 2) < MT;
             const uint16_t* xlane = P.x + static_cast<size_t>(lane >> 2) * P.K + 64 * (lane & 3);
+            // staged x: token min(g, M-1) of the shared copy (see tile_mma_full_s)
+            const uint32_t xs_lane =
+                smem_addr(xs) + static_cast<uint32_t>((min(lane >> 2, P.M - 1) * P.K + 64 * (lane & 3)) * 2);
             while (t < tend) {
                 if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
                     if (lane == 0) atomicExch(s.err, kDevErrTimeout);
@@ -601,7 +714,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 for (int j = 0; j < C; ++j) {
                     if (j < nt) {
                         const int klen = kt == NKT - 1 ? last_len : kKT;
-                        if (P.uniform) {
+                        if (P.uniform && stage) {
+                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2));
+                        } else if (P.uniform) {
                             tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, xrow);
                         } else {
                             tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P);
@@ -611,7 +726,10 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                             float sum[4];
 #pragma unroll
                             for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
-                            finish_group<I8>(P, Z, sum, g, rows, z, t0, t1, lane);
+                            if (!finish_group<I8>(P, s, Z, sum, g, rows, z, t0, t1, lane)) {
+                                if (lane == 0) atomicCAS(s.err, 0, kDevErrTimeout);
+                                dead = true;
+                            }
 #pragma unroll
                             for (int q = 0; q < 4; ++q)
 #pragma unroll
@@ -625,8 +743,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                         }
                     }
                 }
+                // Every lane's reads of the slot have returned (their values fed the MMAs above), so
+                // lane 0 may let the bulk copy overwrite it, as a consumer release would.
                 __syncwarp();
-                if (lane == 0) fence_proxy_async_smem();   // this warp's reads of the slot precede its refill
                 cslot = (cslot + 1 == S) ? 0 : cslot + 1;
                 cphase ^= (cslot == 0) ? 1u : 0u;
                 if (!issue_next()) --in_flight;
@@ -640,6 +759,10 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 }
                 in_flight = 0;
             }
+        }
+        if (stage) {
+            __syncwarp();
+            if (lane == 0) fence_proxy_async_smem();   // this warp's reads of xs precede the next staging
         }
         if (s.nproj > 1 && p + 1 < s.nproj) cta_arrive(&cta_sync[0], &s.done[p], lane);
     }
@@ -657,7 +780,8 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
 // Same per-warp ring and slot size as the stream kernel, no arithmetic: each warp streams a
 // contiguous range of 4 KB pages in slot-sized copies and folds word (lane * 32) of every page
 // into *out.  Measures the read ceiling of the bulk-copy ring.
-__global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* buf, long long pages, unsigned* out) {
+__global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* buf, long long pages, unsigned* out, const unsigned* cw,
+                                                            unsigned long long* rec) {
     constexpr int kPage = 4096, kPagesPerSlot = kSlotBytes / kPage;
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -665,13 +789,15 @@ __global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* b
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kRingBytesPerWarp) + warp * kMaxStages;
     const long long Z = static_cast<long long>(gridDim.x) * kWarps;
     const long long z = static_cast<long long>(blockIdx.x) * kWarps + warp;
-    const long long p0 = z * pages / Z, p1 = (z + 1) * pages / Z;
+    const long long p0 = seg_start(cw, z, static_cast<int>(Z), pages);
+    const long long p1 = seg_start(cw, z + 1, static_cast<int>(Z), pages);
     if (lane == 0) {
         for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     __syncwarp();
     const uint64_t pol = policy_evict_first();
+    const uint64_t tstart = globaltimer_ns();
     long long ip = p0;        // next page to issue
     int islot = 0, in_flight = 0;
     auto issue = [&]() -> bool {
@@ -710,7 +836,13 @@ __global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* b
         if (!issue()) --in_flight;
     }
     for (int o = 16; o; o >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) atomicXor(out, acc);
+    if (lane == 0) {
+        atomicXor(out, acc);
+        if (rec) {
+            rec[2 * z] = tstart;
+            rec[2 * z + 1] = globaltimer_ns();
+        }
+    }
 }
 
 using StreamFn = void (*)(const StreamArgs);
@@ -774,8 +906,9 @@ cudaError_t occupancy(bool i8, int M, int* blocks_per_sm) {
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, f, kThreads, kSmemBytes);
 }
 
-cudaError_t launch_probe(const void* buf, long long chunks, unsigned* out, int grid, cudaStream_t s) {
-    aio_probe_kernel<<<grid, kThreads, kSmemBytes, s>>>(static_cast<const uint8_t*>(buf), chunks, out);
+cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s,
+                         const unsigned* cw, unsigned long long* rec) {
+    aio_probe_kernel<<<grid, kThreads, kSmemBytes, s>>>(static_cast<const uint8_t*>(buf), pages, out, cw, rec);
     return cudaGetLastError();
 }
 

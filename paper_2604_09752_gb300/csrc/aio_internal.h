@@ -27,23 +27,31 @@ constexpr int kStages = kRingBytesPerWarp / kSlotBytes;  // ring slots per warp
 constexpr int kMaxStages = kStages;
 static_assert(kSlotBytes % 4096 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
 constexpr int kSyncOffset = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;  // CTA-level sync words
-constexpr int kSmemBytes = kSyncOffset + 16;
+constexpr int kXsOffset = kSyncOffset + 32;        // sync words (16 B), the x barrier (8 B), padding
+constexpr int kXsBytes = 32 * 1024;                // x staged in shared memory when M * K * 2 fits
+constexpr int kSmemBytes = kXsOffset + kXsBytes;
 constexpr int kMaxM = 8;
 static_assert(kSmemBytes <= 227 * 1024, "ring does not fit in shared memory");
+static_assert(kXsOffset % 16 == 0, "bulk-copy destination alignment");
+
+// Balanced partition: warp z streams tiles [seg(z), seg(z+1)) with seg(z) = (T * cw[z]) >> kCwShift
+// for a nondecreasing per-warp table cw[0..Z] (cw[0] = 0, cw[Z] = 1 << kCwShift).  Without a table
+// seg(z) = z * T / Z.  Either way the warps' segments tile [0, T) exactly.
+constexpr int kCwShift = 20;
 
 constexpr int kDevErrTimeout = 1;       // a bulk-copy wait expired
 constexpr int kDevErrGridTimeout = 2;   // a wait for the previous projection expired
 
 // One projection of a launch; read-only while the kernel runs.  Geometry:
 //   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles;
-//   warp z of the Z warps in the grid streams tiles [z*T/Z, (z+1)*T/Z) of every projection.
+//   warp z of the Z warps in the grid streams tiles [seg(z), seg(z+1)) of every projection.
 struct ProjDesc {
     const uint16_t* x;        // [M, K] bf16
     const uint8_t* w;         // packed (or row-major) weights
     const uint16_t* scales;   // [N] bf16 (int8 only)
     float* y;                 // [M, N] fp32
-    float* partial;           // [Z][2][kRows * M] partial sums of row groups split between warps
-    unsigned* counters;       // [NG] tiles accumulated per split row group; zero between launches
+    float* partial;           // [Z][kRows * M] partial sums of split row groups; 0xFF bytes when empty
+    const void* reserved;     // keeps the descriptor a multiple of 16 bytes
     long long T;
     int K, N, NG, NKT;
     int rowmajor;             // 1: W is row-major [N, K]
@@ -57,6 +65,7 @@ static_assert(sizeof(ProjDesc) % 16 == 0, "descriptor array stride");
 struct StreamArgs {
     const ProjDesc* projs;
     ProjDesc one;
+    const unsigned* cw;       // [Z + 1] cumulative warp weights, or null for equal shares
     unsigned* done;           // [nproj] CTAs finished per projection (nproj > 1 only)
     unsigned* exit_count;     // CTAs that have left the kernel (nproj > 1 only)
     int* err;                 // device error word
@@ -73,14 +82,19 @@ struct Geometry {
 };
 
 Geometry geometry(int K, int N, int num_sms);
-size_t workspace_bytes(const Geometry& g, int M);   // partial sums + counters, 256-B aligned parts
-void carve_workspace(void* base, const Geometry& g, int M, float** partial, unsigned** counters);
+// Partial-sum slots of one launch: Z * kRows * M floats, rounded up to 256 bytes.  Every slot
+// must hold the empty pattern (all bytes 0xFF) when a launch starts; a launch that completes
+// without a device error leaves them so.
+size_t workspace_bytes(const Geometry& g, int M);
 
 cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared memory)
 // pdl: programmatic dependent launch; coop: cooperative launch (all CTAs co-resident).
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop);
 cudaError_t occupancy(bool i8, int M, int* blocks_per_sm);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
-cudaError_t launch_probe(const void* buf, long long chunks, unsigned* out, int grid, cudaStream_t s);
+// Read probe over `pages` 4 KB pages; cw partitions pages like tiles (null: equal shares); rec, if
+// not null, receives per warp z the %globaltimer at start and end: rec[2z], rec[2z+1].
+cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s,
+                         const unsigned* cw = nullptr, unsigned long long* rec = nullptr);
 
 }  // namespace aio

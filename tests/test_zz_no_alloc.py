@@ -78,7 +78,7 @@ def test_noalloc_matches_linear_run(aio, wt, K, N, M, rowmajor):
     aio.aio_linear_destroy(h)
 
 
-def test_noalloc_rejects_oversize_and_bad_arguments(aio):
+def test_noalloc_rejects_oversize_and_bad_arguments(aio, monkeypatch):
     K, N = 256, 64
     x, W, _ = _inputs(K, N, 1, "bf16")
     xd, Wd = _dev(x), _dev(W)
@@ -88,7 +88,6 @@ def test_noalloc_rejects_oversize_and_bad_arguments(aio):
     base = dict(x=xd.data_ptr(), M=1, K=K, N=N, wt=bf, flags=0, W=Wd.data_ptr(), scales=None,
                 y=y.data_ptr(), device_error=err.data_ptr(), stream=0)
     cases = [
-        (dict(N=1 << 24), aio.AIO_ERR_INVALID_ARG, "scratch"),    # counters alone exceed the static scratch
         (dict(M=9), aio.AIO_ERR_INVALID_ARG, None),
         (dict(K=17), aio.AIO_ERR_INVALID_ARG, None),
         (dict(device_error=None), aio.AIO_ERR_INVALID_ARG, None),
@@ -105,6 +104,12 @@ def test_noalloc_rejects_oversize_and_bad_arguments(aio):
         assert e.value.status == code, (over, str(e.value))
         if word:
             assert word in str(e.value)
+    # beyond the static scratch: every M <= 8 fits a GB300's 1 MiB, so the test lowers the limit
+    monkeypatch.setenv("AIO_TEST_NOALLOC_BYTES", "4096")
+    with pytest.raises(aio.AioError) as e:
+        aio.aio_linear_run_noalloc(**base)
+    assert e.value.status == aio.AIO_ERR_INVALID_ARG and "scratch" in str(e.value)
+    monkeypatch.delenv("AIO_TEST_NOALLOC_BYTES")
     torch.cuda.synchronize()
     assert torch.all(y == 7.0), "a rejected call launched work"
     assert err.item() == 0
