@@ -3,7 +3,6 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
-#include <cmath>
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
@@ -72,133 +71,6 @@ aio_status current_device(int* dev, int* sms) {
     return AIO_OK;
 }
 
-// ---------------------------------------------------------------------------------------------
-// Balanced partition.  Under full load the SMs of a GB300 do not stream at one rate: for equal
-// shares some finish up to a third later than others, the same SMs every time (the spread follows
-// the chip's layout, not the data).  In a decode step every projection ends at a grid-wide
-// barrier, so equal shares leave the fast SMs idle at every barrier.  Once per device we measure
-// how long each CTA of a full-grid read takes and move the CTAs' shares toward equal finish times
-// (a few rounds, each rescaling a CTA's weight by mean time / its time).  The table is fixed for
-// the life of the process, so results stay deterministic run to run.  Shares are keyed by CTA
-// index, so the partition is correct whatever SM a CTA lands on; only its balance depends on it.
-// AIO_BALANCE=0 in the environment keeps equal shares.
-std::mutex g_bal_mu;
-bool g_bal_done[64] = {};
-const unsigned* g_bal_cw[64] = {};
-float g_bal_spread[64][2] = {};       // max/min CTA time for equal shares, and for the final table
-
-void cw_from_weights(const std::vector<double>& w, int warps, std::vector<unsigned>& cw) {
-    const int Z = static_cast<int>(w.size()) * warps;
-    double total = 0;
-    for (double v : w) total += v;
-    cw.assign(Z + 1, 0u);
-    double acc = 0;
-    for (int z = 0; z < Z; ++z) {
-        cw[z] = static_cast<unsigned>(std::llround(acc / total * static_cast<double>(1u << aio::kCwShift)));
-        acc += w[z / warps] / warps;
-    }
-    cw[Z] = 1u << aio::kCwShift;
-    for (int z = 1; z <= Z; ++z) cw[z] = std::max(cw[z], cw[z - 1]);
-}
-
-// Per-CTA time of one full-grid read of `bytes` under table cw (null: equal shares), in seconds.
-bool probe_cta_times(const void* buf, size_t bytes, int sms, const unsigned* cw, unsigned* out,
-                     unsigned long long* rec, std::vector<unsigned long long>& h, std::vector<double>& t) {
-    const int Z = sms * aio::kWarps;
-    for (int rep = 0; rep < 2; ++rep)
-        if (aio::launch_probe(buf, static_cast<long long>(bytes / 4096), out, sms, nullptr, cw, rec) != cudaSuccess)
-            return false;
-    if (cudaDeviceSynchronize() != cudaSuccess) return false;
-    h.resize(2 * static_cast<size_t>(Z));
-    if (cudaMemcpy(h.data(), rec, h.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) != cudaSuccess)
-        return false;
-    unsigned long long t0 = ~0ull;
-    for (int z = 0; z < Z; ++z) {
-        if (h[2 * z] == 0 || h[2 * z + 1] < h[2 * z]) return false;
-        t0 = std::min(t0, h[2 * z]);
-    }
-    t.assign(sms, 0.0);
-    for (int z = 0; z < Z; ++z)
-        t[z / aio::kWarps] = std::max(t[z / aio::kWarps], static_cast<double>(h[2 * z + 1] - t0) * 1e-9);
-    return true;
-}
-
-// Builds (once) the calibrated table of the current device `dev`; leaves null (equal shares) when
-// disabled or when the measurement cannot be made.  Synchronises the device.
-void balance_table(int dev, int sms, const unsigned** out) {
-    std::lock_guard<std::mutex> lk(g_bal_mu);
-    if (g_bal_done[dev]) {
-        *out = g_bal_cw[dev];
-        return;
-    }
-    g_bal_done[dev] = true;
-    *out = nullptr;
-    const char* env = getenv("AIO_BALANCE");
-    if (env && env[0] == '0') return;
-    const int Z = sms * aio::kWarps;
-    const size_t cw_bytes = round_up(sizeof(unsigned) * (Z + 1), 256);
-    unsigned* table = nullptr;
-    if (cudaMalloc(&table, cw_bytes) != cudaSuccess) {
-        cudaGetLastError();
-        return;
-    }
-    void* scratch = nullptr;
-    const size_t rec_bytes = round_up(sizeof(unsigned long long) * 2 * Z, 256);
-    size_t bytes = size_t(1) << 30;
-    while (bytes >= (size_t(256) << 20) && cudaMalloc(&scratch, bytes + rec_bytes + 256) != cudaSuccess) {
-        cudaGetLastError();
-        scratch = nullptr;
-        bytes /= 2;
-    }
-    if (!scratch) {
-        cudaFree(table);
-        return;
-    }
-    uint8_t* base = static_cast<uint8_t*>(scratch);
-    auto* rec = reinterpret_cast<unsigned long long*>(base + bytes);
-    auto* xo = reinterpret_cast<unsigned*>(base + bytes + rec_bytes);
-    std::vector<unsigned long long> h;
-    std::vector<double> t, w(sms, 1.0), best_w;
-    std::vector<unsigned> cw;
-    double best = 1e30;
-    bool ok = probe_cta_times(base, bytes, sms, nullptr, xo, rec, h, t);   // warm-up and equal shares
-    if (ok) ok = probe_cta_times(base, bytes, sms, nullptr, xo, rec, h, t);
-    if (ok) {
-        const auto mm = std::minmax_element(t.begin(), t.end());
-        g_bal_spread[dev][0] = static_cast<float>(*mm.second / *mm.first);
-    }
-    for (int it = 0; ok && it < 5; ++it) {
-        double mean = 0;
-        for (double v : t) mean += v / sms;
-        for (int b = 0; b < sms; ++b) w[b] = std::min(2.0, std::max(0.5, w[b] * mean / t[b]));
-        cw_from_weights(w, aio::kWarps, cw);
-        ok = cudaMemcpy(table, cw.data(), sizeof(unsigned) * (Z + 1), cudaMemcpyHostToDevice) == cudaSuccess &&
-             probe_cta_times(base, bytes, sms, table, xo, rec, h, t);
-        if (!ok) break;
-        const auto mm = std::minmax_element(t.begin(), t.end());
-        if (*mm.second < best) {
-            best = *mm.second;
-            best_w = w;
-            g_bal_spread[dev][1] = static_cast<float>(*mm.second / *mm.first);
-        }
-    }
-    if (ok && !best_w.empty()) {
-        cw_from_weights(best_w, aio::kWarps, cw);
-        ok = cudaMemcpy(table, cw.data(), sizeof(unsigned) * (Z + 1), cudaMemcpyHostToDevice) == cudaSuccess;
-    }
-    cudaFree(scratch);
-    if (!ok || best_w.empty()) {
-        cudaGetLastError();
-        cudaFree(table);
-        return;
-    }
-    g_bal_cw[dev] = table;
-    *out = table;
-    if (getenv("AIO_BALANCE_LOG"))
-        fprintf(stderr, "libaio: device %d balance: CTA time spread %.3f with equal shares, %.3f calibrated\n", dev,
-                g_bal_spread[dev][0], g_bal_spread[dev][1]);
-}
-
 aio_status check_device(int dev) {
     int cur = -1;
     AIO_CUDA(cudaGetDevice(&cur));
@@ -237,7 +109,6 @@ struct aio_linear {
     size_t ws_bytes;
     float* partial;      // partial-sum slots (empty pattern 0xFF at rest)
     int* err;
-    const unsigned* cw;  // the device's balanced partition table (null: equal shares)
 };
 
 struct aio_step {
@@ -293,7 +164,6 @@ aio::StreamArgs single_args(const aio_linear* h, const aio::ProjDesc& d, int M, 
     a.nproj = 1;
     a.M = M;
     a.Z = h->geo.Z;
-    a.cw = h->cw;
     a.test_stall = (h->flags & AIO_FLAG_TEST_STALL) ? 1 : 0;
     a.wait_limit_ns = a.test_stall ? kTestWaitLimitNs : kWaitLimitNs;
     return a;
@@ -348,8 +218,6 @@ aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int 
     if (st != AIO_OK) return st;
     aio::Geometry geo = aio::geometry(K, N, sms);
     const size_t ws = aio::workspace_bytes(geo, max_M);
-    const unsigned* cw = nullptr;
-    balance_table(dev, sms, &cw);
     if (test_alloc_failure()) return fail(AIO_ERR_OOM, "workspace allocation failed (AIO_TEST_FAIL_ALLOC)");
     void* mem = nullptr;
     if (cudaMalloc(&mem, ws + 256) != cudaSuccess) {
@@ -378,7 +246,6 @@ aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int 
     h->ws_bytes = ws + 256;
     h->partial = static_cast<float*>(mem);
     h->err = reinterpret_cast<int*>(static_cast<uint8_t*>(mem) + ws);
-    h->cw = cw;
     *out = h;
     return AIO_OK;
 }
@@ -593,7 +460,6 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     w.nproj = n_projs;
     w.M = M;
     w.Z = projs[0].h->geo.Z;
-    w.cw = projs[0].h->cw;
     w.test_stall = 0;
     w.wait_limit_ns = kWaitLimitNs;
     s->whole = w;

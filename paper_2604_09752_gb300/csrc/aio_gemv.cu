@@ -257,10 +257,7 @@ __device__ __forceinline__ void issue_chunk(const ProjDesc* d, int t, int nt, ui
 
 // A warp's walk over its tiles of every projection, one chunk (<= C consecutive tiles) at a time.
 // First tile of warp z's segment of a projection with T tiles (z = Z gives T).
-__device__ __forceinline__ long long seg_start(const unsigned* cw, long long z, int Z, long long T) {
-    if (cw) return (T * static_cast<long long>(__ldg(cw + z))) >> kCwShift;
-    return z * T / Z;
-}
+__device__ __forceinline__ long long seg_start(long long z, int Z, long long T) { return z * T / Z; }
 
 struct ChunkCursor {
     int p, t, te;
@@ -269,8 +266,8 @@ struct ChunkCursor {
 __device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, long long z, int Z) {
     const long long T = proj_desc(s, 0)->T;
     c.p = 0;
-    c.t = static_cast<int>(seg_start(s.cw, z, Z, T));
-    c.te = static_cast<int>(seg_start(s.cw, z + 1, Z, T));
+    c.t = static_cast<int>(seg_start(z, Z, T));
+    c.te = static_cast<int>(seg_start(z + 1, Z, T));
 }
 
 // Next chunk of the walk: its projection, first tile and tile count; false at the end.
@@ -280,8 +277,8 @@ __device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s,
         if (c.p + 1 >= s.nproj) return false;
         ++c.p;
         const long long T = proj_desc(s, c.p)->T;
-        c.t = static_cast<int>(seg_start(s.cw, z, Z, T));
-        c.te = static_cast<int>(seg_start(s.cw, z + 1, Z, T));
+        c.t = static_cast<int>(seg_start(z, Z, T));
+        c.te = static_cast<int>(seg_start(z + 1, Z, T));
     }
     p = c.p;
     t = c.t;
@@ -411,11 +408,11 @@ __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* t
 }
 
 // The same with x staged in shared memory: xaddr is the shared-window address of this lane's
-// x piece 0 for the tile (token min(g, M-1), k = 256 kt + 64c); W and x both come in with
-// ld.shared.v4.  Lanes with g >= M load a real token's x: they fill rows of A whose outputs
-// (tokens >= M) are never written, so no select is needed.
+// x piece 0 for the tile (token g, k = 256 kt + 64c); W and x both come in with ld.shared.v4.
+// Only the lanes of real tokens load x (the 4 lanes of a token read 4 pieces that share banks,
+// so extra lanes would add conflicted wavefronts).
 template <bool I8>
-__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr) {
+__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr, bool xrow) {
     using TL = TileT<I8>;
     constexpr int NP = TL::kPieces;
     uint4 w[NP];
@@ -423,7 +420,7 @@ __device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr
     for (int j = 0; j < NP; ++j) w[j] = lds128(waddr + j * 512);
     uint4 xv[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) xv[j] = lds128(xaddr + 16 * j);
+    for (int j = 0; j < 8; ++j) xv[j] = xrow ? lds128(xaddr + 16 * j) : make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
     for (int s = 0; s < 16; ++s) {
         const uint4& xq = xv[s >> 1];
@@ -498,7 +495,7 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
     // The owner: this warp holds tile gfirst.  The other contributors are the next warps up to the
     // owner of tile tl (segments are contiguous and in warp order).
     long long zl = z;
-    while (zl + 1 < Z && seg_start(s.cw, zl + 1, Z, P.T) <= tl) ++zl;
+    while (zl + 1 < Z && seg_start(zl + 1, Z, P.T) <= tl) ++zl;
     bool ok = true;
     for (int v0 = 0; v0 < V; v0 += 32) {
         const int v = v0 + lane;
@@ -509,7 +506,7 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
         if (v < V && r < rows) {
             float sum = (r & 1) ? own1 : own0;
             for (long long zz = z + 1; ok && zz <= zl; ++zz) {
-                if (seg_start(s.cw, zz + 1, Z, P.T) == seg_start(s.cw, zz, Z, P.T)) continue;   // empty segment
+                if (seg_start(zz + 1, Z, P.T) == seg_start(zz, Z, P.T)) continue;   // empty segment
                 float* slot = P.partial + static_cast<size_t>(zz) * V + v;
                 uint32_t bits = ld_relaxed_u32(slot);
                 if (bits == kSlotEmpty) {
@@ -650,7 +647,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     bool dead = false;    // set after a timeout: stop consuming, keep signalling
     for (int p = 0; p < s.nproj; ++p) {
         Proj P = load_proj(proj_desc(s, p), MT);
-        const long long t0 = seg_start(s.cw, z, Z, P.T), t1 = seg_start(s.cw, z + 1, Z, P.T);
+        const long long t0 = seg_start(z, Z, P.T), t1 = seg_start(z + 1, Z, P.T);
         const uint32_t xbytes = static_cast<uint32_t>(P.M) * static_cast<uint32_t>(P.K) * 2u;
         const bool stage = xbytes <= static_cast<uint32_t>(kXsBytes);
         // Warp 0 stages x once every CTA has finished the previous projection (every warp of this
@@ -699,9 +696,8 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             int rows = min(kRows, P.N - g * kRows);
             const bool xrow = (lane >> 2) < MT;
             const uint16_t* xlane = P.x + static_cast<size_t>(lane >> 2) * P.K + 64 * (lane & 3);
-            // staged x: token min(g, M-1) of the shared copy (see tile_mma_full_s)
-            const uint32_t xs_lane =
-                smem_addr(xs) + static_cast<uint32_t>((min(lane >> 2, P.M - 1) * P.K + 64 * (lane & 3)) * 2);
+            // staged x: the same element offset in the shared copy (rows >= M are never read)
+            const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>(((lane >> 2) * P.K + 64 * (lane & 3)) * 2);
             while (t < tend) {
                 if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
                     if (lane == 0) atomicExch(s.err, kDevErrTimeout);
@@ -715,7 +711,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                     if (j < nt) {
                         const int klen = kt == NKT - 1 ? last_len : kKT;
                         if (P.uniform && stage) {
-                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2));
+                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), xrow);
                         } else if (P.uniform) {
                             tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, xrow);
                         } else {
@@ -780,8 +776,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
 // Same per-warp ring and slot size as the stream kernel, no arithmetic: each warp streams a
 // contiguous range of 4 KB pages in slot-sized copies and folds word (lane * 32) of every page
 // into *out.  Measures the read ceiling of the bulk-copy ring.
-__global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* buf, long long pages, unsigned* out, const unsigned* cw,
-                                                            unsigned long long* rec) {
+__global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* buf, long long pages, unsigned* out) {
     constexpr int kPage = 4096, kPagesPerSlot = kSlotBytes / kPage;
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -789,15 +784,14 @@ __global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* b
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kRingBytesPerWarp) + warp * kMaxStages;
     const long long Z = static_cast<long long>(gridDim.x) * kWarps;
     const long long z = static_cast<long long>(blockIdx.x) * kWarps + warp;
-    const long long p0 = seg_start(cw, z, static_cast<int>(Z), pages);
-    const long long p1 = seg_start(cw, z + 1, static_cast<int>(Z), pages);
+    const long long p0 = seg_start(z, static_cast<int>(Z), pages);
+    const long long p1 = seg_start(z + 1, static_cast<int>(Z), pages);
     if (lane == 0) {
         for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     __syncwarp();
     const uint64_t pol = policy_evict_first();
-    const uint64_t tstart = globaltimer_ns();
     long long ip = p0;        // next page to issue
     int islot = 0, in_flight = 0;
     auto issue = [&]() -> bool {
@@ -836,13 +830,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_probe_kernel(const uint8_t* b
         if (!issue()) --in_flight;
     }
     for (int o = 16; o; o >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) {
-        atomicXor(out, acc);
-        if (rec) {
-            rec[2 * z] = tstart;
-            rec[2 * z + 1] = globaltimer_ns();
-        }
-    }
+    if (lane == 0) atomicXor(out, acc);
 }
 
 using StreamFn = void (*)(const StreamArgs);
@@ -906,9 +894,8 @@ cudaError_t occupancy(bool i8, int M, int* blocks_per_sm) {
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, f, kThreads, kSmemBytes);
 }
 
-cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s,
-                         const unsigned* cw, unsigned long long* rec) {
-    aio_probe_kernel<<<grid, kThreads, kSmemBytes, s>>>(static_cast<const uint8_t*>(buf), pages, out, cw, rec);
+cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s) {
+    aio_probe_kernel<<<grid, kThreads, kSmemBytes, s>>>(static_cast<const uint8_t*>(buf), pages, out);
     return cudaGetLastError();
 }
 

@@ -34,17 +34,12 @@ constexpr int kMaxM = 8;
 static_assert(kSmemBytes <= 227 * 1024, "ring does not fit in shared memory");
 static_assert(kXsOffset % 16 == 0, "bulk-copy destination alignment");
 
-// Balanced partition: warp z streams tiles [seg(z), seg(z+1)) with seg(z) = (T * cw[z]) >> kCwShift
-// for a nondecreasing per-warp table cw[0..Z] (cw[0] = 0, cw[Z] = 1 << kCwShift).  Without a table
-// seg(z) = z * T / Z.  Either way the warps' segments tile [0, T) exactly.
-constexpr int kCwShift = 20;
-
 constexpr int kDevErrTimeout = 1;       // a bulk-copy wait expired
 constexpr int kDevErrGridTimeout = 2;   // a wait for the previous projection expired
 
 // One projection of a launch; read-only while the kernel runs.  Geometry:
 //   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles;
-//   warp z of the Z warps in the grid streams tiles [seg(z), seg(z+1)) of every projection.
+//   warp z of the Z warps in the grid streams tiles [z*T/Z, (z+1)*T/Z) of every projection.
 struct ProjDesc {
     const uint16_t* x;        // [M, K] bf16
     const uint8_t* w;         // packed (or row-major) weights
@@ -65,7 +60,6 @@ static_assert(sizeof(ProjDesc) % 16 == 0, "descriptor array stride");
 struct StreamArgs {
     const ProjDesc* projs;
     ProjDesc one;
-    const unsigned* cw;       // [Z + 1] cumulative warp weights, or null for equal shares
     unsigned* done;           // [nproj] CTAs finished per projection (nproj > 1 only)
     unsigned* exit_count;     // CTAs that have left the kernel (nproj > 1 only)
     int* err;                 // device error word
@@ -92,9 +86,6 @@ cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared 
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop);
 cudaError_t occupancy(bool i8, int M, int* blocks_per_sm);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
-// Read probe over `pages` 4 KB pages; cw partitions pages like tiles (null: equal shares); rec, if
-// not null, receives per warp z the %globaltimer at start and end: rec[2z], rec[2z+1].
-cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s,
-                         const unsigned* cw = nullptr, unsigned long long* rec = nullptr);
+cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s);
 
 }  // namespace aio
