@@ -79,10 +79,14 @@ typedef enum {
                                       this flag the step is a chain of one launch per projection. */
 
 /* Packed weight layout written by aio_linear_pack (a permutation of W, no padding):
- * rows are grouped 8 at a time and each group is cut into tiles of 256 k-columns;
- * tile (g, kt) starts at element 8*g*K + rows_g*256*kt, rows_g = min(8, N - 8g), and is
- * the row-major block W[8g : 8g+rows_g, 256kt : 256kt+len], len = min(256, K - 256kt). */
-#define AIO_ROWS_PER_GROUP 8
+ * rows are grouped 16 at a time and each group is cut into tiles of 256 k-columns;
+ * tile (g, kt) starts at element 16*g*K + rows_g*256*kt, rows_g = min(16, N - 16g), and holds
+ * the block W[16g : 16g+rows_g, 256kt : 256kt+len], len = min(256, K - 256kt): row-major when
+ * ragged (rows_g < 16 or len < 256), otherwise in the stream kernel's fragment order (16-byte
+ * piece j of lane L = 4r + c at byte j*512 + 16L holds runs of 8 consecutive k,
+ * W[row][32t + 8c : 32t + 8c + 8], t = 0..7; bf16: piece j = 8h + t is row r + 8h, run t;
+ * int8: piece j = 4h + u is row r + 8h, runs t = 2u then 2u + 1). */
+#define AIO_ROWS_PER_GROUP 16
 #define AIO_K_TILE 256
 
 typedef struct aio_linear* aio_linear_t;
@@ -168,9 +172,9 @@ aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, co
  *   device_error  device int, 4-byte aligned, owned by the caller: set non-zero if a bounded
  *                 device-side wait expired (y is then incomplete); the library never clears it
  * Scratch: the cross-warp partial sums live in one static device array of
- * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs 256 M S
+ * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs 512 M S
  * bytes of it (S = the device's SM count), rounded up to 256: on a 152-SM GB300 every M <= 8 fits
- * (311296 bytes at M = 8).  A call that needs more returns AIO_ERR_INVALID_ARG and launches nothing.
+ * (622592 bytes at M = 8).  A call that needs more returns AIO_ERR_INVALID_ARG and launches nothing.
  * Each call enqueues a cudaMemsetAsync that empties the partial-sum slots it uses (all bytes 0xFF),
  * then the kernel.
  * Every call on a device shares that scratch: calls that overlap in time race and give wrong

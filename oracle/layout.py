@@ -5,15 +5,17 @@ is one contiguous block of bytes, and so that a full tile sits in shared memory 
 kernel's lanes read it.  The layout is a pure permutation of the elements, written here with
 plain numpy slicing so the GPU packer can be checked bit for bit against it:
 
-  * rows are grouped 8 at a time: row group g holds rows [8g, 8g + rows_g),
-    rows_g = min(8, N - 8g); the group starts at element offset 8 g K;
+  * rows are grouped 16 at a time: row group g holds rows [16g, 16g + rows_g),
+    rows_g = min(16, N - 16g); the group starts at element offset 16 g K;
   * inside a group, k is cut into tiles of 256 columns: tile kt covers
     [256 kt, 256 kt + len_kt), len_kt = min(256, K - 256 kt), and starts at
     element offset rows_g * 256 * kt from the start of its group;
-  * a full tile (rows_g = 8, len_kt = 256) is stored as 16-byte pieces: piece j of lane
-    L = 4 r + c (r = row in the tile, c = 0..3) holds the P consecutive elements
-    W[r, 64 c + P j : 64 c + P (j + 1)] (P = 8 for 2-byte, 16 for 1-byte elements) and sits at
-    byte j * 512 + L * 16 of the tile;
+  * a full tile (rows_g = 16, len_kt = 256) is stored as 16-byte pieces, 32 lanes per piece
+    index: lane L = 4 r + c (r = 0..7, c = 0..3) reads piece j at byte j * 512 + 16 L of the
+    tile.  Its pieces hold runs of 8 consecutive k, W[row, 32 t + 8 c : 32 t + 8 c + 8]:
+      - 2-byte elements: piece j (0..15) is row r + 8 (j // 8), run t = j % 8;
+      - 1-byte elements: piece j (0..7) is row r + 8 (j // 4), runs t = 2 (j % 4) then
+        2 (j % 4) + 1 (8 bytes each);
   * a ragged tile is the row-major block [rows_g, len_kt].
 
 No padding is added, so the packed buffer has exactly N*K elements.
@@ -22,7 +24,7 @@ from __future__ import annotations
 
 import numpy as np
 
-ROWS_PER_GROUP = 8
+ROWS_PER_GROUP = 16
 K_TILE = 256
 
 
@@ -31,17 +33,28 @@ def tile_offset(N: int, K: int, g: int, kt: int) -> int:
     return ROWS_PER_GROUP * g * K + rows_g * K_TILE * kt
 
 
+def _lane_runs(esize: int, j: int, L: int):
+    """The (row, first k) of the 8-element runs that piece j of lane L holds, in storage order."""
+    r, c = divmod(L, 4)
+    if esize == 2:
+        per_half = K_TILE // 32                  # pieces of one row per lane
+        return [(r + 8 * (j // per_half), 32 * (j % per_half) + 8 * c)]
+    per_half = K_TILE // 64
+    u = j % per_half
+    row = r + 8 * (j // per_half)
+    return [(row, 32 * (2 * u) + 8 * c), (row, 32 * (2 * u + 1) + 8 * c)]
+
+
 def _full_tile_order(esize: int) -> np.ndarray:
     """order[i] = row-major index (r * 256 + k) of the element stored at position i of a full tile."""
-    P = 16 // esize                      # elements per 16-byte piece
-    pieces = 256 // (4 * P)              # pieces per lane
+    pieces = ROWS_PER_GROUP * K_TILE * esize // 512      # 16-byte pieces per lane
     order = np.empty(ROWS_PER_GROUP * K_TILE, dtype=np.int64)
     for j in range(pieces):
         for L in range(32):
-            r, c = divmod(L, 4)
             pos = (j * 512 + L * 16) // esize
-            k0 = 64 * c + P * j
-            order[pos:pos + P] = r * K_TILE + k0 + np.arange(P)
+            for row, k0 in _lane_runs(esize, j, L):
+                order[pos:pos + 8] = row * K_TILE + k0 + np.arange(8)
+                pos += 8
     return order
 
 

@@ -39,7 +39,7 @@ AIO_FLAG_TEST_STALL = 0x100
 AIO_STEP_GRAPH = 0x1
 AIO_STEP_PDL = 0x2
 AIO_STEP_PERSISTENT = 0x4
-AIO_ROWS_PER_GROUP = 8
+AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
 for _name, _val in re.findall(r"#define\s+(AIO_\w+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", _hdr):

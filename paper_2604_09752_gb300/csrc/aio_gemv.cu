@@ -5,7 +5,7 @@
 // The work is a stream of weight bytes from HBM with 1 (bf16) or 2 (int8) multiply-adds per byte per
 // token row.  Design:
 //
-//   * Tiles.  W is cut into tiles of 8 rows x 256 k (4 KB bf16, 2 KB int8); consecutive tiles are
+//   * Tiles.  W is cut into tiles of 16 rows x 256 k (8 KB bf16, 4 KB int8); consecutive tiles are
 //     contiguous in the packed layout, so any run of them is one bulk copy.  The T tiles of a matrix
 //     are split evenly over the Z warps of the grid: warp z streams tiles [z*T/Z, (z+1)*T/Z), so
 //     every warp moves the same bytes to within one tile whatever N and K are.
@@ -13,18 +13,16 @@
 //     cp.async.bulk per slot (global -> shared, L2 evict-first) completing on the slot's mbarrier;
 //     the warp waits (bounded by %globaltimer), computes, and refills the slot.  The issue cursor
 //     runs ahead across projection boundaries: weights never depend on x.
-//   * Arithmetic on the tensor cores.  For the 16-k step s of a tile, lane (g, c) = (lane/4, lane%4)
-//     supplies x[token g][64c + 4s + 0..3] as its A fragment (rows 8..15 of A are zero) and
-//     W[row g][64c + 4s + 0..3] as its B fragment of one mma.sync.m16n8k16 (bf16 in, fp32
-//     accumulate).  This assignment of the 256 k of a tile to (s, c, position) is a permutation
-//     shared by A and B, so the sum is unchanged; it makes each lane's 64 W elements and 64 x
-//     elements of a tile contiguous.  Full tiles are stored in fragment order ([j][lane][16 B]),
-//     so the W loads are conflict-free 128-bit shared loads.  D[token g][row 2c, 2c+1] lands in
-//     lane (g, c): the k-reduction across lanes is done by the MMA, and the work per byte does not
-//     grow with M.  k-step s accumulates into one of four chains (s % 4) to keep MMAs in flight.
-//     int8 codes become bf16 exactly (|q| <= 128 fits bf16's 8 significant bits) with two bit
-//     operations and one bf16x2 subtraction per pair; the per-channel scale multiplies the
-//     finished fp32 sum.
+//   * x.  Once per CTA and projection, warp 0 stages x into shared memory (one bulk copy per token
+//     row, rows padded by 64 B) when it fits; otherwise the lanes read x from global memory.
+//   * Arithmetic on the tensor cores: mma.sync.m16n8k16, bf16 in, fp32 accumulate, with A = W
+//     (the tile's 16 rows) and B = x (up to 8 tokens), so one MMA reduces 256 weights for every
+//     token and the work per byte does not grow with M.  A k-permutation shared by A and B (see
+//     tile_mma_frag) gives each lane runs of 8 consecutive k; full tiles are stored in fragment
+//     order ([j][lane][16 B]), so W comes in with conflict-free 128-bit shared loads.  Four
+//     accumulator chains keep MMAs in flight.  int8 codes become bf16 exactly (|q| <= 128 fits
+//     bf16's 8 significant bits) with two bit operations and one bf16x2 subtraction per pair; the
+//     per-channel scale multiplies the finished fp32 sum.
 //   * Split row groups.  A row group whose tiles all lie in one warp's segment is written directly.
 //     A group split between warps is owned by its first contributor, for which it is the last group
 //     of its segment, so the owner reaches it at the end of the phase; the other contributors reach
@@ -185,10 +183,9 @@ __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_floa
 template <bool I8>
 struct TileT {
     static constexpr int kEsize = I8 ? 1 : 2;
-    static constexpr int kBytes = kRows * kKT * kEsize;    // 2048 or 4096
+    static constexpr int kBytes = kRows * kKT * kEsize;    // 4096 (int8) or 8192 (bf16)
     static constexpr int kChunk = kSlotBytes / kBytes;     // tiles per ring slot
-    static constexpr int kPieces = kBytes / 512;           // 16-byte pieces per lane per tile (4 or 8)
-    static constexpr int kPieceElems = 16 / kEsize;        // elements per piece (16 or 8)
+    static constexpr int kPieces = kBytes / 512;           // 16-byte pieces per lane per tile (8 or 16)
 };
 
 __device__ __forceinline__ const ProjDesc* proj_desc(const StreamArgs& s, int p) {
@@ -314,17 +311,60 @@ __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
     return p;
 }
 
-// One tile: D += x[:, k-range] * W[rows, k-range]^T on the tensor cores.  Lane (g, c) loads its 16
-// k-steps' worth of W (row g) and x (token g), each 64 contiguous k starting at 64c.  Full packed
-// tiles use the fragment-ordered layout; ragged tiles (rows < 8 or klen < 256) and row-major
-// weights are row-major, and any piece outside the tile (or a token >= M) is zero.  k-step s
-// accumulates into d[s % 4], so four MMA chains are in flight instead of one.
+// ------------------------------------------------------------------ one tile on the tensor cores
+// A tile is 16 rows x 256 k of W.  It takes 16 k-steps of mma.m16n8k16 with A = W (lane (g, c)
+// supplies rows g and g + 8 of the tile) and B = x (lane (g, c) supplies token g), so one MMA
+// reduces 256 weights for all M <= 8 tokens at once; D[row][token] accumulates in fp32.
+// k-permutation: in k-step s, lane (g, c) holds the logical k pairs (2c, 2c+1) and (2c+8, 2c+9)
+// of both operands, which are the physical k = 32(s/2) + 8c + 4(s%2) + {0, 1} and + {2, 3}.
+// The map is a bijection onto the tile's 256 k and A and B share it, so the sum is unchanged.
+// Per pair of k-steps t = s/2 a lane therefore reads 8 consecutive k at 32t + 8c of W rows g and
+// g + 8 and of x token g; the four lanes of a token read 64 consecutive bytes of x (no shared-
+// memory bank conflict).  k-step s accumulates into d[s % 4]: four MMA chains in flight.
+constexpr int kRuns = kKT / 32;   // runs of 8 k per lane and row: x pieces per tile, bf16 pieces per row half
+
+template <bool I8>
+__device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)[TileT<I8>::kPieces],
+                                              const uint4 (&xv)[kRuns]) {
+#pragma unroll
+    for (int s = 0; s < kKT / 16; ++s) {
+        const int t = s >> 1, q = s & 1;
+        const uint4& xq = xv[t];
+        const uint32_t b0 = q ? xq.z : xq.x;
+        const uint32_t b1 = q ? xq.w : xq.y;
+        uint32_t a0, a1, a2, a3;
+        if constexpr (I8) {
+            // piece t/2 of row g (kRuns/2 + t/2 of row g + 8); word 2(t%2) + q holds the step's 4 codes
+            const uint4& lo = w[t >> 1];
+            const uint4& hi = w[kRuns / 2 + (t >> 1)];
+            const int wi = (t & 1) * 2 + q;
+            const uint32_t wl = wi == 0 ? lo.x : wi == 1 ? lo.y : wi == 2 ? lo.z : lo.w;
+            const uint32_t wh = wi == 0 ? hi.x : wi == 1 ? hi.y : wi == 2 ? hi.z : hi.w;
+            a0 = i8x2_to_bf16x2<0x4140u>(wl);
+            a2 = i8x2_to_bf16x2<0x4342u>(wl);
+            a1 = i8x2_to_bf16x2<0x4140u>(wh);
+            a3 = i8x2_to_bf16x2<0x4342u>(wh);
+        } else {
+            const uint4& lo = w[t];
+            const uint4& hi = w[kRuns + t];
+            a0 = q ? lo.z : lo.x;
+            a2 = q ? lo.w : lo.y;
+            a1 = q ? hi.z : hi.x;
+            a3 = q ? hi.w : hi.y;
+        }
+        mma_bf16(d[s & 3], a0, a1, a2, a3, b0, b1);
+    }
+}
+
+// Any tile: full packed tiles in fragment order (piece j at j * 512 + 16 lane); ragged tiles
+// (rows < 16 or klen < 256) and row-major weights as the row-major block [rows][klen].  Pieces
+// outside the tile are zero, and so is x outside [kbase, kbase + klen) or for tokens >= M.
+// x is read from xp = x + token g's row (row stride xstride elements), staged or global.
 template <bool I8>
 __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, int rows, int klen, int kbase,
-                                         int lane, const Proj& P) {
+                                         int lane, const Proj& P, const uint16_t* xrow_ptr) {
     using TL = TileT<I8>;
-    constexpr int NP = TL::kPieces;          // 16-byte W pieces per lane
-    constexpr int PE = TL::kPieceElems;      // elements per W piece
+    constexpr int NP = TL::kPieces;
     const int g = lane >> 2, c = lane & 3;
     const bool full = rows == kRows && klen == kKT && !P.rowmajor;
     uint4 w[NP];
@@ -332,113 +372,59 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
     for (int j = 0; j < NP; ++j) {
         if (full) {
             w[j] = *reinterpret_cast<const uint4*>(tile + j * 512 + lane * 16);
+        } else if constexpr (I8) {
+            // piece j: row g + 8 (j / (kRuns/2)), runs t = 2 (j % (kRuns/2)) and t + 1, 8 codes each
+            const int r = g + 8 * (j / (kRuns / 2)), ka = 64 * (j % (kRuns / 2)) + 8 * c, kb = ka + 32;
+            const uint8_t* rowp = tile + static_cast<size_t>(r) * klen;
+            const uint2 lo = (r < rows && ka < klen) ? *reinterpret_cast<const uint2*>(rowp + ka) : make_uint2(0u, 0u);
+            const uint2 hi = (r < rows && kb < klen) ? *reinterpret_cast<const uint2*>(rowp + kb) : make_uint2(0u, 0u);
+            w[j] = make_uint4(lo.x, lo.y, hi.x, hi.y);
         } else {
-            const int k = 64 * c + PE * j;
-            if (g < rows && k < klen)
-                w[j] = *reinterpret_cast<const uint4*>(tile + (static_cast<size_t>(g) * klen + k) * TL::kEsize);
-            else
-                w[j] = make_uint4(0u, 0u, 0u, 0u);
+            // piece j: row g + 8 (j / kRuns), run t = j % kRuns
+            const int r = g + 8 * (j / kRuns), k = 32 * (j % kRuns) + 8 * c;
+            w[j] = (r < rows && k < klen)
+                       ? *reinterpret_cast<const uint4*>(tile + (static_cast<size_t>(r) * klen + k) * 2)
+                       : make_uint4(0u, 0u, 0u, 0u);
         }
     }
-    // x: 64 bf16 of token g starting at kbase + 64c, as 8 pieces of 8
-    uint4 xv[8];
+    uint4 xv[kRuns];
     const bool xrow = g < P.M;
-    const uint16_t* xp = P.x + static_cast<size_t>(g) * P.K + kbase + 64 * c;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        if (xrow && 64 * c + 8 * j < klen)
-            xv[j] = *reinterpret_cast<const uint4*>(xp + 8 * j);
-        else
-            xv[j] = make_uint4(0u, 0u, 0u, 0u);
+    for (int t = 0; t < kRuns; ++t) {
+        const int k = 32 * t + 8 * c;
+        xv[t] = (xrow && k < klen) ? *reinterpret_cast<const uint4*>(xrow_ptr + kbase + k) : make_uint4(0u, 0u, 0u, 0u);
     }
-    // k-step s covers elements 4s..4s+3 of the lane's 64: x piece s/2, words 2(s%2), 2(s%2)+1
-#pragma unroll
-    for (int s = 0; s < 16; ++s) {
-        const uint4& xq = xv[s >> 1];
-        const uint32_t a0 = (s & 1) ? xq.z : xq.x;
-        const uint32_t a2 = (s & 1) ? xq.w : xq.y;
-        uint32_t b0, b1;
-        if constexpr (I8) {
-            // W piece s/4 holds codes 16*(s/4) .. +15; k-step s uses word s%4 (4 codes)
-            const uint4& wq = w[s >> 2];
-            const uint32_t word = (s & 3) == 0 ? wq.x : (s & 3) == 1 ? wq.y : (s & 3) == 2 ? wq.z : wq.w;
-            b0 = i8x2_to_bf16x2<0x4140u>(word);
-            b1 = i8x2_to_bf16x2<0x4342u>(word);
-        } else {
-            const uint4& wq = w[s >> 1];
-            b0 = (s & 1) ? wq.z : wq.x;
-            b1 = (s & 1) ? wq.w : wq.y;
-        }
-        mma_bf16(d[s & 3], a0, 0u, a2, 0u, b0, b1);
-    }
+    tile_mma_frag<I8>(d, w, xv);
 }
 
-// The same for a full packed tile, with no bounds logic: W pieces at j * 512 + lane * 16 of the
-// tile, x pieces at xp + 8j (xp = x + token * K + 256 kt + 64c), x zero for tokens >= M.
+// A full packed tile with x in global memory: xp = x + token g's row + 256 kt + 8c; x is zero for
+// tokens >= M.
 template <bool I8>
 __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp,
                                               bool xrow) {
     using TL = TileT<I8>;
-    constexpr int NP = TL::kPieces;
-    uint4 w[NP];
+    uint4 w[TL::kPieces];
 #pragma unroll
-    for (int j = 0; j < NP; ++j) w[j] = *reinterpret_cast<const uint4*>(tile_lane + j * 512);
-    uint4 xv[8];
+    for (int j = 0; j < TL::kPieces; ++j) w[j] = *reinterpret_cast<const uint4*>(tile_lane + j * 512);
+    uint4 xv[kRuns];
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-        xv[j] = xrow ? *reinterpret_cast<const uint4*>(xp + 8 * j) : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int s = 0; s < 16; ++s) {
-        const uint4& xq = xv[s >> 1];
-        const uint32_t a0 = (s & 1) ? xq.z : xq.x;
-        const uint32_t a2 = (s & 1) ? xq.w : xq.y;
-        uint32_t b0, b1;
-        if constexpr (I8) {
-            const uint4& wq = w[s >> 2];
-            const uint32_t word = (s & 3) == 0 ? wq.x : (s & 3) == 1 ? wq.y : (s & 3) == 2 ? wq.z : wq.w;
-            b0 = i8x2_to_bf16x2<0x4140u>(word);
-            b1 = i8x2_to_bf16x2<0x4342u>(word);
-        } else {
-            const uint4& wq = w[s >> 1];
-            b0 = (s & 1) ? wq.z : wq.x;
-            b1 = (s & 1) ? wq.w : wq.y;
-        }
-        mma_bf16(d[s & 3], a0, 0u, a2, 0u, b0, b1);
-    }
+    for (int t = 0; t < kRuns; ++t) xv[t] = xrow ? *reinterpret_cast<const uint4*>(xp + 32 * t) : make_uint4(0u, 0u, 0u, 0u);
+    tile_mma_frag<I8>(d, w, xv);
 }
 
-// The same with x staged in shared memory: xaddr is the shared-window address of this lane's
-// x piece 0 for the tile (token g, k = 256 kt + 64c); W and x both come in with ld.shared.v4.
-// Only the lanes of real tokens load x (the 4 lanes of a token read 4 pieces that share banks,
-// so extra lanes would add conflicted wavefronts).
+// A full packed tile with x staged in shared memory: waddr / xaddr are shared-window addresses of
+// this lane's piece 0 of W and of x (token g, k = 256 kt + 8c); both come in with ld.shared.v4.
+// Only the lanes of real tokens load x: the others would only add wavefronts.
 template <bool I8>
 __device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr, bool xrow) {
     using TL = TileT<I8>;
-    constexpr int NP = TL::kPieces;
-    uint4 w[NP];
+    uint4 w[TL::kPieces];
 #pragma unroll
-    for (int j = 0; j < NP; ++j) w[j] = lds128(waddr + j * 512);
-    uint4 xv[8];
+    for (int j = 0; j < TL::kPieces; ++j) w[j] = lds128(waddr + j * 512);
+    uint4 xv[kRuns];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) xv[j] = xrow ? lds128(xaddr + 16 * j) : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-    for (int s = 0; s < 16; ++s) {
-        const uint4& xq = xv[s >> 1];
-        const uint32_t a0 = (s & 1) ? xq.z : xq.x;
-        const uint32_t a2 = (s & 1) ? xq.w : xq.y;
-        uint32_t b0, b1;
-        if constexpr (I8) {
-            const uint4& wq = w[s >> 2];
-            const uint32_t word = (s & 3) == 0 ? wq.x : (s & 3) == 1 ? wq.y : (s & 3) == 2 ? wq.z : wq.w;
-            b0 = i8x2_to_bf16x2<0x4140u>(word);
-            b1 = i8x2_to_bf16x2<0x4342u>(word);
-        } else {
-            const uint4& wq = w[s >> 1];
-            b0 = (s & 1) ? wq.z : wq.x;
-            b1 = (s & 1) ? wq.w : wq.y;
-        }
-        mma_bf16(d[s & 3], a0, 0u, a2, 0u, b0, b1);
-    }
+    for (int t = 0; t < kRuns; ++t) xv[t] = xrow ? lds128(xaddr + 64 * t) : make_uint4(0u, 0u, 0u, 0u);
+    tile_mma_frag<I8>(d, w, xv);
 }
 
 template <bool I8>
@@ -458,24 +444,24 @@ __device__ __forceinline__ uint32_t slot_bits(float v) {
     return v != v ? 0x7FC00000u : __float_as_uint(v);
 }
 
-// Warp z has finished its tiles of row group g: lane (g', c) holds D[token g'][rows 2c, 2c+1].
-// Writes y (group complete in this warp), stores the partial (split group, not the owner), or, as
-// the owner, adds the other contributors' partials and writes y.  Returns false if a wait for a
-// partial expired or the launch already failed.
+// Warp z has finished its tiles of row group g: lane (g', c) holds d = D[row g'][token 2c],
+// D[row g'][token 2c + 1], D[row g' + 8][token 2c], D[row g' + 8][token 2c + 1].  Writes y (group
+// complete in this warp), stores the partial (split group, not the owner), or, as the owner, adds
+// the other contributors' partials and writes y.  Returns false if a wait for a partial expired or
+// the launch already failed.
 template <bool I8>
 __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s, int Z, const float (&d)[4], int g,
                                              int rows, long long z, long long t0, long long t1, int lane) {
-    const int tok = lane >> 2, r0 = 2 * (lane & 3);
+    const int gr = lane >> 2, m0 = 2 * (lane & 3);
     const int row0 = g * kRows;
     const long long gfirst = static_cast<long long>(g) * P.NKT;
     const long long tl = gfirst + P.NKT - 1;
-    const bool mine = tok < P.M;
 
     if (t0 <= gfirst && t1 > tl) {
-        if (mine) {
-            float* yp = P.y + static_cast<size_t>(tok) * P.N + row0 + r0;
-            if (r0 < rows) yp[0] = d[0] * row_scale<I8>(P, row0 + r0);
-            if (r0 + 1 < rows) yp[1] = d[1] * row_scale<I8>(P, row0 + r0 + 1);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int m = m0 + (i & 1), r = gr + 8 * (i >> 1);
+            if (m < P.M && r < rows) P.y[static_cast<size_t>(m) * P.N + row0 + r] = d[i] * row_scale<I8>(P, row0 + r);
         }
         return true;
     }
@@ -485,9 +471,10 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
         // Not the owner: g is this warp's first group (its last split group it always owns), so
         // one slot per warp suffices.  Publish [token][row] and go on.
         float* part = P.partial + static_cast<size_t>(z) * V;
-        if (mine) {
-            st_relaxed_u32(part + tok * kRows + r0, slot_bits(d[0]));
-            st_relaxed_u32(part + tok * kRows + r0 + 1, slot_bits(d[1]));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int m = m0 + (i & 1), r = gr + 8 * (i >> 1);
+            if (m < P.M) st_relaxed_u32(part + m * kRows + r, slot_bits(d[i]));
         }
         return true;
     }
@@ -500,23 +487,34 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
     for (int v0 = 0; v0 < V; v0 += 32) {
         const int v = v0 + lane;
         const int m = v / kRows, r = v - m * kRows;
-        const int src = (m * 4 + (r >> 1)) & 31;          // the lane holding the owner's own value
-        const float own0 = __shfl_sync(0xffffffffu, d[0], src);
-        const float own1 = __shfl_sync(0xffffffffu, d[1], src);
+        const int src = ((r & 7) * 4 + (m >> 1)) & 31;   // the lane holding the owner's own value
+        const int idx = (r >> 3) * 2 + (m & 1);
+        const float o0 = __shfl_sync(0xffffffffu, d[0], src), o1 = __shfl_sync(0xffffffffu, d[1], src);
+        const float o2 = __shfl_sync(0xffffffffu, d[2], src), o3 = __shfl_sync(0xffffffffu, d[3], src);
         if (v < V && r < rows) {
-            float sum = (r & 1) ? own1 : own0;
-            for (long long zz = z + 1; ok && zz <= zl; ++zz) {
-                if (seg_start(zz + 1, Z, P.T) == seg_start(zz, Z, P.T)) continue;   // empty segment
-                float* slot = P.partial + static_cast<size_t>(zz) * V + v;
-                uint32_t bits = ld_relaxed_u32(slot);
-                if (bits == kSlotEmpty) {
-                    const uint64_t start = globaltimer_ns();
-                    while (ok && (bits = ld_relaxed_u32(slot)) == kSlotEmpty)
-                        ok = ld_relaxed_u32(s.err) == 0u && globaltimer_ns() - start <= s.wait_limit_ns;
-                }
-                if (ok) {
-                    sum += __uint_as_float(bits);
-                    st_relaxed_u32(slot, kSlotEmpty);
+            float sum = idx == 0 ? o0 : idx == 1 ? o1 : idx == 2 ? o2 : o3;
+            // Four contributors at a time: their slots are loaded together (independent loads, one
+            // round trip), then added in warp order; only slots still empty are polled.
+            for (long long zb = z + 1; ok && zb <= zl; zb += 4) {
+                uint32_t bits[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    bits[i] = zb + i <= zl ? ld_relaxed_u32(P.partial + static_cast<size_t>(zb + i) * V + v) : 0u;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const long long zz = zb + i;
+                    if (!ok || zz > zl) break;
+                    if (seg_start(zz + 1, Z, P.T) == seg_start(zz, Z, P.T)) continue;   // empty segment
+                    float* slot = P.partial + static_cast<size_t>(zz) * V + v;
+                    if (bits[i] == kSlotEmpty) {
+                        const uint64_t start = globaltimer_ns();
+                        while (ok && (bits[i] = ld_relaxed_u32(slot)) == kSlotEmpty)
+                            ok = ld_relaxed_u32(s.err) == 0u && globaltimer_ns() - start <= s.wait_limit_ns;
+                    }
+                    if (ok) {
+                        sum += __uint_as_float(bits[i]);
+                        st_relaxed_u32(slot, kSlotEmpty);
+                    }
                 }
             }
             if (ok) P.y[static_cast<size_t>(m) * P.N + row0 + r] = sum * row_scale<I8>(P, row0 + r);
@@ -648,14 +646,19 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     for (int p = 0; p < s.nproj; ++p) {
         Proj P = load_proj(proj_desc(s, p), MT);
         const long long t0 = seg_start(z, Z, P.T), t1 = seg_start(z + 1, Z, P.T);
-        const uint32_t xbytes = static_cast<uint32_t>(P.M) * static_cast<uint32_t>(P.K) * 2u;
-        const bool stage = xbytes <= static_cast<uint32_t>(kXsBytes);
+        // Staged x rows are kXsPad elements apart beyond K, so two tokens read in one shared-memory
+        // phase fall in different banks.
+        const int xs_stride = P.K + kXsPad;
+        const bool stage = P.M * xs_stride * 2 <= kXsBytes;
         // Warp 0 stages x once every CTA has finished the previous projection (every warp of this
-        // CTA has then finished reading the previous x and fenced its reads against async writes).
+        // CTA has then finished reading the previous x and fenced its reads against async writes):
+        // one bulk copy per token row.
         auto stage_x = [&]() {
             if (stage && lane == 0) {
-                mbar_expect_tx(xbar, xbytes);
-                bulk_g2s_plain(xs, P.x, xbytes, xbar);
+                mbar_expect_tx(xbar, static_cast<uint32_t>(P.M * P.K * 2));
+                for (int m = 0; m < P.M; ++m)
+                    bulk_g2s_plain(xs + m * xs_stride, P.x + static_cast<size_t>(m) * P.K,
+                                   static_cast<uint32_t>(P.K * 2), xbar);
             }
         };
         if (p == 0 && warp == 0) stage_x();
@@ -684,7 +687,6 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 dead = true;
             }
             xphase ^= 1u;
-            P.x = xs;   // the general tile path reads the staged copy too
         }
         if (!dead && t1 > t0) {
             float d[4][4] = {};
@@ -694,10 +696,12 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             const int tend = static_cast<int>(t1);
             int g = t / NKT, kt = t - g * NKT;
             int rows = min(kRows, P.N - g * kRows);
-            const bool xrow = (lane >> 2) < MT;
-            const uint16_t* xlane = P.x + static_cast<size_t>(lane >> 2) * P.K + 64 * (lane & 3);
-            // staged x: the same element offset in the shared copy (rows >= M are never read)
-            const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>(((lane >> 2) * P.K + 64 * (lane & 3)) * 2);
+            const int tok = lane >> 2;
+            const bool xrow = tok < MT;
+            // x of this lane's token (rows >= M are never read): the staged copy or global memory
+            const uint16_t* xrow_ptr = stage ? xs + tok * xs_stride : P.x + static_cast<size_t>(tok) * P.K;
+            const uint16_t* xlane = P.x + static_cast<size_t>(tok) * P.K + 8 * (lane & 3);
+            const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>((tok * xs_stride + 8 * (lane & 3)) * 2);
             while (t < tend) {
                 if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
                     if (lane == 0) atomicExch(s.err, kDevErrTimeout);
@@ -715,7 +719,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                         } else if (P.uniform) {
                             tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, xrow);
                         } else {
-                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P);
+                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr);
                         }
                         tp += rows * klen * E;
                         if (kt == NKT - 1 || t == tend - 1) {

@@ -17,7 +17,7 @@
 
 namespace aio {
 
-constexpr int kRows = 8;                    // rows per row group (AIO_ROWS_PER_GROUP)
+constexpr int kRows = 16;                   // rows per row group (AIO_ROWS_PER_GROUP)
 constexpr int kKT = 256;                    // k columns per tile (AIO_K_TILE)
 constexpr int kWarps = AIO_WARPS;           // every warp streams its own tile segment
 constexpr int kThreads = kWarps * 32;
@@ -28,7 +28,8 @@ constexpr int kMaxStages = kStages;
 static_assert(kSlotBytes % 4096 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
 constexpr int kSyncOffset = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;  // CTA-level sync words
 constexpr int kXsOffset = kSyncOffset + 32;        // sync words (16 B), the x barrier (8 B), padding
-constexpr int kXsBytes = 32 * 1024;                // x staged in shared memory when M * K * 2 fits
+constexpr int kXsPad = 32;                         // elements between staged x rows beyond K (64 B)
+constexpr int kXsBytes = 227 * 1024 - kXsOffset;   // x staged in shared memory when M * (K + kXsPad) * 2 fits
 constexpr int kSmemBytes = kXsOffset + kXsBytes;
 constexpr int kMaxM = 8;
 static_assert(kSmemBytes <= 227 * 1024, "ring does not fit in shared memory");

@@ -1,11 +1,14 @@
 // aio_pack.cu -- weight packer: row-major W [N, K] <-> tiled layout.
 //
-// Tiles are 8 rows x 256 k; consecutive tiles are contiguous, so any run of them is one bulk copy.
-// A full tile (8 rows, 256 k) is stored in the order the stream kernel's lanes read it: 16-byte
-// piece j of lane L = 4 r + c holds W[row r][64 c + j * (8 bf16 | 16 int8) ...], at byte
-// j * 512 + L * 16 of the tile, so every 128-bit shared-memory load of a warp is contiguous.
-// Ragged tiles (last row group or last k tile) stay row-major.  The layout is a pure permutation
-// (no padding); one thread moves one 16-byte piece, and the row-major side is fully coalesced.
+// Tiles are 16 rows x 256 k; consecutive tiles are contiguous, so any run of them is one bulk copy.
+// A full tile (16 rows, 256 k) is stored in the order the stream kernel's lanes read it: lane
+// L = 4 r + c (r = 0..7, c = 0..3) reads 16-byte piece j at byte j * 512 + 16 L of the tile, and
+// its pieces hold runs of 8 consecutive k, W[row][32 t + 8 c .. +8), t = 0..7:
+//   bf16: piece j = 8 h + t holds row r + 8 h, run t;
+//   int8: piece j = 4 h + u holds row r + 8 h, runs t = 2u (bytes 0-7) and t = 2u + 1 (bytes 8-15).
+// Every 128-bit shared-memory load of a warp is then contiguous.  Ragged tiles (last row group or
+// last k tile) stay row-major.  The layout is a pure permutation (no padding); one thread moves one
+// 8-byte unit, and the row-major side is fully coalesced.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -17,13 +20,13 @@ namespace {
 template <int E, bool INVERSE>
 __global__ void __launch_bounds__(256) aio_pack_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
                                                        int N, int K) {
-    constexpr int kPiece = 16 / E;                 // elements per 16-byte piece
-    const long long per_row = K / kPiece;
+    constexpr int kUnit = 8 / E;                   // elements per 8-byte unit
+    const long long per_row = K / kUnit;
     const long long total = static_cast<long long>(N) * per_row;
     for (long long p = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; p < total;
          p += static_cast<long long>(gridDim.x) * blockDim.x) {
         const int n = static_cast<int>(p / per_row);
-        const int k = static_cast<int>(p - static_cast<long long>(n) * per_row) * kPiece;
+        const int k = static_cast<int>(p - static_cast<long long>(n) * per_row) * kUnit;
         const int g = n / kRows, r = n - g * kRows;
         const int kt = k / kKT, kk = k - kt * kKT;
         const int rows = min(kRows, N - g * kRows);
@@ -31,17 +34,21 @@ __global__ void __launch_bounds__(256) aio_pack_kernel(const uint8_t* __restrict
         const size_t tile = (static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT) * E;
         size_t in_tile;
         if (rows == kRows && klen == kKT) {
-            const int c = kk / 64, j = (kk - 64 * c) / kPiece;
-            in_tile = static_cast<size_t>(j) * 512 + (r * 4 + c) * 16;
+            const int h = r >> 3, lane = (r & 7) * 4 + ((kk & 31) >> 3), t = kk >> 5;
+            if (E == 2) {
+                in_tile = static_cast<size_t>((kKT / 32) * h + t) * 512 + lane * 16 + (kk & 7) * 2;
+            } else {
+                in_tile = static_cast<size_t>((kKT / 64) * h + (t >> 1)) * 512 + lane * 16 + (t & 1) * 8;
+            }
         } else {
             in_tile = (static_cast<size_t>(r) * klen + kk) * E;
         }
         const size_t packed = tile + in_tile;
         const size_t rowmajor = (static_cast<size_t>(n) * K + k) * E;
         if (INVERSE) {
-            *reinterpret_cast<uint4*>(dst + rowmajor) = *reinterpret_cast<const uint4*>(src + packed);
+            *reinterpret_cast<uint2*>(dst + rowmajor) = *reinterpret_cast<const uint2*>(src + packed);
         } else {
-            *reinterpret_cast<uint4*>(dst + packed) = *reinterpret_cast<const uint4*>(src + rowmajor);
+            *reinterpret_cast<uint2*>(dst + packed) = *reinterpret_cast<const uint2*>(src + rowmajor);
         }
     }
 }
@@ -49,9 +56,9 @@ __global__ void __launch_bounds__(256) aio_pack_kernel(const uint8_t* __restrict
 }  // namespace
 
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s) {
-    const long long pieces = static_cast<long long>(N) * K * esize / 16;
+    const long long units = static_cast<long long>(N) * K * esize / 8;
     const int block = 256;
-    long long grid = (pieces + block - 1) / block;
+    long long grid = (units + block - 1) / block;
     if (grid > 65535LL * 16) grid = 65535LL * 16;
     if (grid < 1) grid = 1;
     const uint8_t* a = static_cast<const uint8_t*>(src);
