@@ -145,6 +145,8 @@ aio::ProjDesc make_desc(const aio_linear* h, const void* x, const void* W, const
     d.y = y;
     d.partial = partial;
     d.T = h->geo.T;
+    d.Tq = static_cast<int>(h->geo.T / h->geo.Z);
+    d.Tr = static_cast<int>(h->geo.T % h->geo.Z);
     d.K = h->K;
     d.N = h->N;
     d.NG = h->geo.NG;
@@ -650,6 +652,8 @@ extern "C" aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N,
     d.y = y;
     d.partial = partial;
     d.T = geo.T;
+    d.Tq = static_cast<int>(geo.T / geo.Z);
+    d.Tr = static_cast<int>(geo.T % geo.Z);
     d.K = K;
     d.N = N;
     d.NG = geo.NG;

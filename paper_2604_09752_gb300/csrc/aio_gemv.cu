@@ -199,16 +199,41 @@ __device__ __forceinline__ size_t tile_offset(int K, int N, int g, int kt) {
     return (static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT) * E;
 }
 
+// What the issuing lane needs of one projection, held in registers.
+struct IssueProj {
+    const uint8_t* w;
+    int Tq, Tr;           // T = Tq * Z + Tr
+    int K, N, NKT;
+    int uniform, rowmajor;
+};
+
+__device__ __forceinline__ IssueProj load_issue(const ProjDesc* d) {
+    IssueProj q;
+    q.w = d->w;
+    q.Tq = d->Tq;
+    q.Tr = d->Tr;
+    q.K = d->K;
+    q.N = d->N;
+    q.NKT = d->NKT;
+    q.uniform = d->uniform;
+    q.rowmajor = d->rowmajor;
+    return q;
+}
+
+// First tile of warp z's segment (z = Z gives T): floor(z T / Z) = z Tq + floor(z Tr / Z), exact in
+// 32-bit arithmetic (z Tq <= T < 2^31 and z Tr < Z^2).
+__device__ __forceinline__ int seg(int z, int Z, int Tq, int Tr) { return z * Tq + (z * Tr) / Z; }
+
 // Lane 0: arm the slot's barrier with the chunk's byte count and issue the copies of tiles
 // [t, t + nt) of projection d.  Packed weights: one bulk copy.  Row-major weights: one copy per
 // tile row, landing in the row-major form of that tile.
 template <bool I8>
-__device__ __noinline__ void issue_chunk_general(const ProjDesc* d, int t, int nt, uint8_t* dst, uint64_t* bar,
+__device__ __noinline__ void issue_chunk_general(IssueProj d, int t, int nt, uint8_t* dst, uint64_t* bar,
                                                  uint64_t pol) {
     constexpr int E = TileT<I8>::kEsize;
-    const int K = d->K, N = d->N, NKT = d->NKT;
+    const int K = d.K, N = d.N, NKT = d.NKT;
     int g = t / NKT, kt = t - g * NKT;
-    if (!d->rowmajor) {
+    if (!d.rowmajor) {
         const int tl = t + nt - 1;
         const int gl = tl / NKT, ktl = tl - gl * NKT;
         const int rows_l = min(kRows, N - gl * kRows), klen_l = min(kKT, K - ktl * kKT);
@@ -216,7 +241,7 @@ __device__ __noinline__ void issue_chunk_general(const ProjDesc* d, int t, int n
         const size_t end = tile_offset<E>(K, N, gl, ktl) + static_cast<size_t>(rows_l) * klen_l * E;
         const uint32_t bytes = static_cast<uint32_t>(end - off);
         mbar_expect_tx(bar, bytes);
-        bulk_g2s(dst, d->w + off, bytes, bar, pol);
+        bulk_g2s(dst, d.w + off, bytes, bar, pol);
         return;
     }
     uint32_t total = 0;
@@ -232,7 +257,7 @@ __device__ __noinline__ void issue_chunk_general(const ProjDesc* d, int t, int n
         const int rows = min(kRows, N - g * kRows), klen = min(kKT, K - kt * kKT);
         for (int r = 0; r < rows; ++r) {
             const size_t off = (static_cast<size_t>(g * kRows + r) * K + static_cast<size_t>(kt) * kKT) * E;
-            bulk_g2s(dst + r * klen * E, d->w + off, static_cast<uint32_t>(klen * E), bar, pol);
+            bulk_g2s(dst + r * klen * E, d.w + off, static_cast<uint32_t>(klen * E), bar, pol);
         }
         dst += rows * klen * E;
         if (++kt == NKT) { kt = 0; ++g; }
@@ -240,42 +265,47 @@ __device__ __noinline__ void issue_chunk_general(const ProjDesc* d, int t, int n
 }
 
 template <bool I8>
-__device__ __forceinline__ void issue_chunk(const ProjDesc* d, int t, int nt, uint8_t* dst, uint64_t* bar,
+__device__ __forceinline__ void issue_chunk(const IssueProj& d, int t, int nt, uint8_t* dst, uint64_t* bar,
                                             uint64_t pol) {
     constexpr int B = TileT<I8>::kBytes;
-    if (d->uniform) {   // every tile full: tile t is bytes [t * B, (t + 1) * B)
+    if (d.uniform) {   // every tile full: tile t is bytes [t * B, (t + 1) * B)
         const uint32_t bytes = static_cast<uint32_t>(nt * B);
         mbar_expect_tx(bar, bytes);
-        bulk_g2s(dst, d->w + static_cast<size_t>(t) * B, bytes, bar, pol);
+        bulk_g2s(dst, d.w + static_cast<size_t>(t) * B, bytes, bar, pol);
         return;
     }
     issue_chunk_general<I8>(d, t, nt, dst, bar, pol);
 }
 
-// A warp's walk over its tiles of every projection, one chunk (<= C consecutive tiles) at a time.
-// First tile of warp z's segment of a projection with T tiles (z = Z gives T).
+// First page of a probe warp's range (64-bit: any buffer size).
 __device__ __forceinline__ long long seg_start(long long z, int Z, long long T) { return z * T / Z; }
 
+// A warp's walk over its tiles of every projection, one chunk (<= C consecutive tiles) at a time.
+// It holds the issue fields of the current projection and, loaded one projection ahead, of the
+// next, so crossing a projection boundary never waits on a descriptor load.
 struct ChunkCursor {
     int p, t, te;
+    IssueProj cur, nxt;
 };
 
-__device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, long long z, int Z) {
-    const long long T = proj_desc(s, 0)->T;
+__device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, int z, int Z) {
+    c.cur = load_issue(proj_desc(s, 0));
+    c.nxt = s.nproj > 1 ? load_issue(proj_desc(s, 1)) : c.cur;
     c.p = 0;
-    c.t = static_cast<int>(seg_start(z, Z, T));
-    c.te = static_cast<int>(seg_start(z + 1, Z, T));
+    c.t = seg(z, Z, c.cur.Tq, c.cur.Tr);
+    c.te = seg(z + 1, Z, c.cur.Tq, c.cur.Tr);
 }
 
 // Next chunk of the walk: its projection, first tile and tile count; false at the end.
-__device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s, long long z, int Z, int C, int& p,
+__device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s, int z, int Z, int C, int& p,
                                             int& t, int& nt) {
     while (c.t >= c.te) {
         if (c.p + 1 >= s.nproj) return false;
         ++c.p;
-        const long long T = proj_desc(s, c.p)->T;
-        c.t = static_cast<int>(seg_start(z, Z, T));
-        c.te = static_cast<int>(seg_start(z + 1, Z, T));
+        c.cur = c.nxt;
+        if (c.p + 1 < s.nproj) c.nxt = load_issue(proj_desc(s, c.p + 1));
+        c.t = seg(z, Z, c.cur.Tq, c.cur.Tr);
+        c.te = seg(z + 1, Z, c.cur.Tq, c.cur.Tr);
     }
     p = c.p;
     t = c.t;
@@ -291,6 +321,7 @@ struct Proj {
     float* y;
     float* partial;
     long long T;
+    int Tq, Tr;
     int M, K, N, NKT;
     int rowmajor, uniform;
 };
@@ -301,6 +332,8 @@ __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
     p.scales = d->scales;
     p.y = d->y;
     p.partial = d->partial;
+    p.Tq = d->Tq;
+    p.Tr = d->Tr;
     p.T = d->T;
     p.M = M;
     p.K = d->K;
@@ -482,7 +515,7 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
     // The owner: this warp holds tile gfirst.  The other contributors are the next warps up to the
     // owner of tile tl (segments are contiguous and in warp order).
     long long zl = z;
-    while (zl + 1 < Z && seg_start(zl + 1, Z, P.T) <= tl) ++zl;
+    while (zl + 1 < Z && seg(static_cast<int>(zl) + 1, Z, P.Tq, P.Tr) <= tl) ++zl;
     bool ok = true;
     for (int v0 = 0; v0 < V; v0 += 32) {
         const int v = v0 + lane;
@@ -504,7 +537,8 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
                 for (int i = 0; i < 4; ++i) {
                     const long long zz = zb + i;
                     if (!ok || zz > zl) break;
-                    if (seg_start(zz + 1, Z, P.T) == seg_start(zz, Z, P.T)) continue;   // empty segment
+                    if (seg(static_cast<int>(zz) + 1, Z, P.Tq, P.Tr) == seg(static_cast<int>(zz), Z, P.Tq, P.Tr))
+                        continue;   // empty segment
                     float* slot = P.partial + static_cast<size_t>(zz) * V + v;
                     if (bits[i] == kSlotEmpty) {
                         const uint64_t start = globaltimer_ns();
@@ -623,7 +657,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         int ip, it, nt;
         if (!cursor_next(ring_cur, s, z, Z, C, ip, it, nt)) return false;
         if (lane == 0 && !(stall && first_issue))   // test hook: this slot's barrier never completes
-            issue_chunk<I8>(proj_desc(s, ip), it, nt, ring + islot * kSlotBytes, &bars[islot], pol);
+            issue_chunk<I8>(ring_cur.cur, it, nt, ring + islot * kSlotBytes, &bars[islot], pol);
         first_issue = false;
         islot = (islot + 1 == S) ? 0 : islot + 1;
         return true;
@@ -645,7 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     bool dead = false;    // set after a timeout: stop consuming, keep signalling
     for (int p = 0; p < s.nproj; ++p) {
         Proj P = load_proj(proj_desc(s, p), MT);
-        const long long t0 = seg_start(z, Z, P.T), t1 = seg_start(z + 1, Z, P.T);
+        const long long t0 = seg(static_cast<int>(z), Z, P.Tq, P.Tr), t1 = seg(static_cast<int>(z) + 1, Z, P.Tq, P.Tr);
         // Staged x rows are kXsPad elements apart beyond K, so two tokens read in one shared-memory
         // phase fall in different banks.
         const int xs_stride = P.K + kXsPad;

@@ -47,7 +47,7 @@ struct ProjDesc {
     const uint16_t* scales;   // [N] bf16 (int8 only)
     float* y;                 // [M, N] fp32
     float* partial;           // [Z][kRows * M] partial sums of split row groups; 0xFF bytes when empty
-    const void* reserved;     // keeps the descriptor a multiple of 16 bytes
+    int Tq, Tr;               // T = Tq * Z + Tr (Z = warps in the grid): segment bounds in 32-bit arithmetic
     long long T;
     int K, N, NG, NKT;
     int rowmajor;             // 1: W is row-major [N, K]
