@@ -430,33 +430,35 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
     tile_mma_frag<I8>(d, w, xv);
 }
 
-// A full packed tile with x in global memory: xp = x + token g's row + 256 kt + 8c; x is zero for
-// tokens >= M.
+// A full packed tile with x in global memory: xp = x + token min(g, M-1)'s row + 256 kt + 8c.
+// Lanes g >= M load a real token's x (the same addresses as lanes of token M-1, served once):
+// they only fill columns of D for tokens >= M, which are never written.  No select is needed.
 template <bool I8>
-__device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp,
-                                              bool xrow) {
+__device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp) {
     using TL = TileT<I8>;
     uint4 w[TL::kPieces];
 #pragma unroll
     for (int j = 0; j < TL::kPieces; ++j) w[j] = *reinterpret_cast<const uint4*>(tile_lane + j * 512);
     uint4 xv[kRuns];
 #pragma unroll
-    for (int t = 0; t < kRuns; ++t) xv[t] = xrow ? *reinterpret_cast<const uint4*>(xp + 32 * t) : make_uint4(0u, 0u, 0u, 0u);
+    for (int t = 0; t < kRuns; ++t) xv[t] = *reinterpret_cast<const uint4*>(xp + 32 * t);
     tile_mma_frag<I8>(d, w, xv);
 }
 
 // A full packed tile with x staged in shared memory: waddr / xaddr are shared-window addresses of
-// this lane's piece 0 of W and of x (token g, k = 256 kt + 8c); both come in with ld.shared.v4.
-// Only the lanes of real tokens load x: the others would only add wavefronts.
+// this lane's piece 0 of W and of x (token min(g, M-1), k = 256 kt + 8c); both come in with
+// ld.shared.v4.  The four lanes of a token read 64 contiguous bytes of x, and lanes g >= M read the
+// same addresses as token M-1's lanes (a broadcast), so the x loads are free of bank conflicts and
+// need no select; those lanes only fill columns of D for tokens >= M, which are never written.
 template <bool I8>
-__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr, bool xrow) {
+__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr) {
     using TL = TileT<I8>;
     uint4 w[TL::kPieces];
 #pragma unroll
     for (int j = 0; j < TL::kPieces; ++j) w[j] = lds128(waddr + j * 512);
     uint4 xv[kRuns];
 #pragma unroll
-    for (int t = 0; t < kRuns; ++t) xv[t] = xrow ? lds128(xaddr + 64 * t) : make_uint4(0u, 0u, 0u, 0u);
+    for (int t = 0; t < kRuns; ++t) xv[t] = lds128(xaddr + 64 * t);
     tile_mma_frag<I8>(d, w, xv);
 }
 
@@ -731,11 +733,11 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             int g = t / NKT, kt = t - g * NKT;
             int rows = min(kRows, P.N - g * kRows);
             const int tok = lane >> 2;
-            const bool xrow = tok < MT;
             // x of this lane's token (rows >= M are never read): the staged copy or global memory
             const uint16_t* xrow_ptr = stage ? xs + tok * xs_stride : P.x + static_cast<size_t>(tok) * P.K;
-            const uint16_t* xlane = P.x + static_cast<size_t>(tok) * P.K + 8 * (lane & 3);
-            const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>((tok * xs_stride + 8 * (lane & 3)) * 2);
+            const int xtok = min(tok, MT - 1);   // full tiles: lanes of tokens >= M read token M-1's x
+            const uint16_t* xlane = P.x + static_cast<size_t>(xtok) * P.K + 8 * (lane & 3);
+            const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>((xtok * xs_stride + 8 * (lane & 3)) * 2);
             while (t < tend) {
                 if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
                     if (lane == 0) atomicExch(s.err, kDevErrTimeout);
@@ -749,9 +751,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                     if (j < nt) {
                         const int klen = kt == NKT - 1 ? last_len : kKT;
                         if (P.uniform && stage) {
-                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), xrow);
+                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2));
                         } else if (P.uniform) {
-                            tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, xrow);
+                            tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT);
                         } else {
                             tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr);
                         }
