@@ -85,7 +85,8 @@ typedef enum {
  * ragged (rows_g < 16 or len < 256), otherwise in the stream kernel's fragment order (16-byte
  * piece j of lane L = 4r + c at byte j*512 + 16L holds runs of 8 consecutive k,
  * W[row][32t + 8c : 32t + 8c + 8], t = 0..7; bf16: piece j = 8h + t is row r + 8h, run t;
- * int8: piece j = 4h + u is row r + 8h, runs t = 2u then 2u + 1). */
+ * int8: piece j = 4h + u is row r + 8h, runs t = 2u then 2u + 1, each 4-code word of a run
+ * stored as codes (0, 2, 1, 3)). */
 #define AIO_ROWS_PER_GROUP 16
 #define AIO_K_TILE 256
 

@@ -15,7 +15,9 @@ plain numpy slicing so the GPU packer can be checked bit for bit against it:
     tile.  Its pieces hold runs of 8 consecutive k, W[row, 32 t + 8 c : 32 t + 8 c + 8]:
       - 2-byte elements: piece j (0..15) is row r + 8 (j // 8), run t = j % 8;
       - 1-byte elements: piece j (0..7) is row r + 8 (j // 4), runs t = 2 (j % 4) then
-        2 (j % 4) + 1 (8 bytes each);
+        2 (j % 4) + 1 (8 bytes each), each run stored as k + (0, 2, 1, 3, 4, 6, 5, 7): in every
+        4-byte word the codes of the first k pair sit in the low bytes of the two 16-bit halves
+        and those of the second pair in the high bytes;
   * a ragged tile is the row-major block [rows_g, len_kt].
 
 No padding is added, so the packed buffer has exactly N*K elements.
@@ -26,6 +28,7 @@ import numpy as np
 
 ROWS_PER_GROUP = 16
 K_TILE = 256
+INT8_RUN_ORDER = np.array([0, 2, 1, 3, 4, 6, 5, 7])   # storage order of an 8-code run in a full int8 tile
 
 
 def tile_offset(N: int, K: int, g: int, kt: int) -> int:
@@ -52,8 +55,9 @@ def _full_tile_order(esize: int) -> np.ndarray:
     for j in range(pieces):
         for L in range(32):
             pos = (j * 512 + L * 16) // esize
+            within = np.arange(8) if esize == 2 else INT8_RUN_ORDER
             for row, k0 in _lane_runs(esize, j, L):
-                order[pos:pos + 8] = row * K_TILE + k0 + np.arange(8)
+                order[pos:pos + 8] = row * K_TILE + k0 + within
                 pos += 8
     return order
 

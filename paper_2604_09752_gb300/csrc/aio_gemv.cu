@@ -165,12 +165,10 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Two int8 codes (the bytes of w selected by SEL) -> bf16x2, exactly.  With t holding the code bytes
-// in the low byte of each 16-bit half: 0x4300 | (q & 0x7F) is bf16 128 + (q & 0x7F), and
-// 0x4300 | (q & 0x80) is bf16 128 or 256; their difference is q.
-template <uint32_t SEL>
-__device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t w) {
-    const uint32_t t = __byte_perm(w, 0u, SEL);
+// Two int8 codes -> bf16x2, exactly.  t holds the codes in the low bytes of its 16-bit halves (the
+// high bytes are ignored): 0x4300 | (q & 0x7F) is bf16 128 + (q & 0x7F), and 0x4300 | (q & 0x80)
+// is bf16 128 or 256; their difference is q.
+__device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t t) {
     const uint32_t a = (t & 0x007F007Fu) | 0x43004300u;
     const uint32_t b = (t & 0x00800080u) | 0x43004300u;
     __nv_bfloat162 r = __hsub2(*reinterpret_cast<const __nv_bfloat162*>(&a),
@@ -367,16 +365,17 @@ __device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)
         const uint32_t b1 = q ? xq.w : xq.y;
         uint32_t a0, a1, a2, a3;
         if constexpr (I8) {
-            // piece t/2 of row g (kRuns/2 + t/2 of row g + 8); word 2(t%2) + q holds the step's 4 codes
+            // piece t/2 of row g (kRuns/2 + t/2 of row g + 8); word 2(t%2) + q holds the step's 4 codes,
+            // stored (0, 2, 1, 3): k pair (0, 1) in the low bytes of its halves, (2, 3) in the high
             const uint4& lo = w[t >> 1];
             const uint4& hi = w[kRuns / 2 + (t >> 1)];
             const int wi = (t & 1) * 2 + q;
             const uint32_t wl = wi == 0 ? lo.x : wi == 1 ? lo.y : wi == 2 ? lo.z : lo.w;
             const uint32_t wh = wi == 0 ? hi.x : wi == 1 ? hi.y : wi == 2 ? hi.z : hi.w;
-            a0 = i8x2_to_bf16x2<0x4140u>(wl);
-            a2 = i8x2_to_bf16x2<0x4342u>(wl);
-            a1 = i8x2_to_bf16x2<0x4140u>(wh);
-            a3 = i8x2_to_bf16x2<0x4342u>(wh);
+            a0 = i8x2_to_bf16x2(wl);
+            a2 = i8x2_to_bf16x2(wl >> 8);
+            a1 = i8x2_to_bf16x2(wh);
+            a3 = i8x2_to_bf16x2(wh >> 8);
         } else {
             const uint4& lo = w[t];
             const uint4& hi = w[kRuns + t];
@@ -411,7 +410,9 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
             const uint8_t* rowp = tile + static_cast<size_t>(r) * klen;
             const uint2 lo = (r < rows && ka < klen) ? *reinterpret_cast<const uint2*>(rowp + ka) : make_uint2(0u, 0u);
             const uint2 hi = (r < rows && kb < klen) ? *reinterpret_cast<const uint2*>(rowp + kb) : make_uint2(0u, 0u);
-            w[j] = make_uint4(lo.x, lo.y, hi.x, hi.y);
+            // row-major codes: put each word in the (0, 2, 1, 3) order full tiles are stored in
+            w[j] = make_uint4(__byte_perm(lo.x, 0u, 0x3120u), __byte_perm(lo.y, 0u, 0x3120u),
+                              __byte_perm(hi.x, 0u, 0x3120u), __byte_perm(hi.y, 0u, 0x3120u));
         } else {
             // piece j: row g + 8 (j / kRuns), run t = j % kRuns
             const int r = g + 8 * (j / kRuns), k = 32 * (j % kRuns) + 8 * c;

@@ -5,7 +5,9 @@
 // L = 4 r + c (r = 0..7, c = 0..3) reads 16-byte piece j at byte j * 512 + 16 L of the tile, and
 // its pieces hold runs of 8 consecutive k, W[row][32 t + 8 c .. +8), t = 0..7:
 //   bf16: piece j = 8 h + t holds row r + 8 h, run t;
-//   int8: piece j = 4 h + u holds row r + 8 h, runs t = 2u (bytes 0-7) and t = 2u + 1 (bytes 8-15).
+//   int8: piece j = 4 h + u holds row r + 8 h, runs t = 2u (bytes 0-7) and t = 2u + 1 (bytes 8-15),
+//         each 4-code word of a run stored as codes (0, 2, 1, 3): the first k pair in the low bytes
+//         of the word's 16-bit halves, the second in the high bytes (the swap is its own inverse).
 // Every 128-bit shared-memory load of a warp is then contiguous.  Ragged tiles (last row group or
 // last k tile) stay row-major.  The layout is a pure permutation (no padding); one thread moves one
 // 8-byte unit, and the row-major side is fully coalesced.
@@ -45,11 +47,12 @@ __global__ void __launch_bounds__(256) aio_pack_kernel(const uint8_t* __restrict
         }
         const size_t packed = tile + in_tile;
         const size_t rowmajor = (static_cast<size_t>(n) * K + k) * E;
-        if (INVERSE) {
-            *reinterpret_cast<uint2*>(dst + rowmajor) = *reinterpret_cast<const uint2*>(src + packed);
-        } else {
-            *reinterpret_cast<uint2*>(dst + packed) = *reinterpret_cast<const uint2*>(src + rowmajor);
+        uint2 v = *reinterpret_cast<const uint2*>(src + (INVERSE ? packed : rowmajor));
+        if (E == 1 && rows == kRows && klen == kKT) {   // swap bytes 1 and 2 of each word
+            v.x = __byte_perm(v.x, 0u, 0x3120u);
+            v.y = __byte_perm(v.y, 0u, 0x3120u);
         }
+        *reinterpret_cast<uint2*>(dst + (INVERSE ? rowmajor : packed)) = v;
     }
 }
 

@@ -82,7 +82,8 @@ def test_full_tile_fragment_order_int8():
              (4, 0): (8, 0, 32), (7, 13): (3 + 8, 192 + 8, 224 + 8)}
     for (j, L), (row, ka, kb) in cases.items():
         pos = j * 512 + L * 16
-        want = [row * T + ka + e for e in range(8)] + [row * T + kb + e for e in range(8)]
+        swz = (0, 2, 1, 3, 4, 6, 5, 7)   # each 4-code word holds k pairs (0,1) in its low bytes, (2,3) in its high bytes
+        want = [row * T + ka + e for e in swz] + [row * T + kb + e for e in swz]
         assert list(order[pos:pos + 16]) == want, (j, L)
 
 
