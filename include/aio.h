@@ -82,11 +82,11 @@ typedef enum {
  * rows are grouped 16 at a time and each group is cut into tiles of 256 k-columns;
  * tile (g, kt) starts at element 16*g*K + rows_g*256*kt, rows_g = min(16, N - 16g), and holds
  * the block W[16g : 16g+rows_g, 256kt : 256kt+len], len = min(256, K - 256kt): row-major when
- * ragged (rows_g < 16 or len < 256), otherwise in the stream kernel's fragment order (16-byte
- * piece j of lane L = 4r + c at byte j*512 + 16L holds runs of 8 consecutive k,
- * W[row][32t + 8c : 32t + 8c + 8], t = 0..7; bf16: piece j = 8h + t is row r + 8h, run t;
- * int8: piece j = 4h + u is row r + 8h, runs t = 2u then 2u + 1, each 4-code word of a run
- * stored as codes (0, 2, 1, 3)). */
+ * ragged (rows_g < 16 or len < 256), otherwise in the stream kernel's fragment order: lane
+ * L = 4r + c reads 16-byte piece j at byte j*512 + 16L.  bf16: piece s holds, with
+ * k0 = 32(s/2) + 8c + 4(s%2), the pairs W[r][k0..k0+1], W[r+8][k0..k0+1], W[r][k0+2..k0+3],
+ * W[r+8][k0+2..k0+3].  int8: piece j = 4h + u holds the 8-code runs W[r+8h][32t + 8c : +8] for
+ * t = 2u then 2u + 1, each 4-code word stored as codes (0, 2, 1, 3). */
 #define AIO_ROWS_PER_GROUP 16
 #define AIO_K_TILE 256
 

@@ -12,9 +12,12 @@ plain numpy slicing so the GPU packer can be checked bit for bit against it:
     element offset rows_g * 256 * kt from the start of its group;
   * a full tile (rows_g = 16, len_kt = 256) is stored as 16-byte pieces, 32 lanes per piece
     index: lane L = 4 r + c (r = 0..7, c = 0..3) reads piece j at byte j * 512 + 16 L of the
-    tile.  Its pieces hold runs of 8 consecutive k, W[row, 32 t + 8 c : 32 t + 8 c + 8]:
-      - 2-byte elements: piece j (0..15) is row r + 8 (j // 8), run t = j % 8;
-      - 1-byte elements: piece j (0..7) is row r + 8 (j // 4), runs t = 2 (j % 4) then
+    tile:
+      - 2-byte elements: piece s (0..15) holds, with k0 = 32 (s // 2) + 8 c + 4 (s % 2), the
+        pairs W[r, k0:k0+2], W[r+8, k0:k0+2], W[r, k0+2:k0+4], W[r+8, k0+2:k0+4] (one MMA's A
+        fragment, in register order);
+      - 1-byte elements: pieces hold runs of 8 consecutive k, W[row, 32 t + 8 c : 32 t + 8 c + 8];
+        piece j (0..7) is row r + 8 (j // 4), runs t = 2 (j % 4) then
         2 (j % 4) + 1 (8 bytes each), each run stored as k + (0, 2, 1, 3, 4, 6, 5, 7): in every
         4-byte word the codes of the first k pair sit in the low bytes of the two 16-bit halves
         and those of the second pair in the high bytes;
@@ -37,15 +40,20 @@ def tile_offset(N: int, K: int, g: int, kt: int) -> int:
 
 
 def _lane_runs(esize: int, j: int, L: int):
-    """The (row, first k) of the 8-element runs that piece j of lane L holds, in storage order."""
+    """int8: the (row, first k) of the 8-code runs that piece j of lane L holds, in storage order."""
     r, c = divmod(L, 4)
-    if esize == 2:
-        per_half = K_TILE // 32                  # pieces of one row per lane
-        return [(r + 8 * (j // per_half), 32 * (j % per_half) + 8 * c)]
     per_half = K_TILE // 64
     u = j % per_half
     row = r + 8 * (j // per_half)
     return [(row, 32 * (2 * u) + 8 * c), (row, 32 * (2 * u + 1) + 8 * c)]
+
+
+def _bf16_piece(s: int, L: int):
+    """(row, k) of the 8 elements of bf16 piece s of lane L, in storage order."""
+    r, c = divmod(L, 4)
+    k0 = 32 * (s // 2) + 8 * c + 4 * (s % 2)
+    return [(r, k0), (r, k0 + 1), (r + 8, k0), (r + 8, k0 + 1),
+            (r, k0 + 2), (r, k0 + 3), (r + 8, k0 + 2), (r + 8, k0 + 3)]
 
 
 def _full_tile_order(esize: int) -> np.ndarray:
@@ -55,9 +63,11 @@ def _full_tile_order(esize: int) -> np.ndarray:
     for j in range(pieces):
         for L in range(32):
             pos = (j * 512 + L * 16) // esize
-            within = np.arange(8) if esize == 2 else INT8_RUN_ORDER
+            if esize == 2:
+                order[pos:pos + 8] = [row * K_TILE + k for row, k in _bf16_piece(j, L)]
+                continue
             for row, k0 in _lane_runs(esize, j, L):
-                order[pos:pos + 8] = row * K_TILE + k0 + within
+                order[pos:pos + 8] = row * K_TILE + k0 + INT8_RUN_ORDER
                 pos += 8
     return order
 

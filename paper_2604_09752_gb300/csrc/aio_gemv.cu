@@ -377,12 +377,11 @@ __device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)
             a1 = i8x2_to_bf16x2(wh);
             a3 = i8x2_to_bf16x2(wh >> 8);
         } else {
-            const uint4& lo = w[t];
-            const uint4& hi = w[kRuns + t];
-            a0 = q ? lo.z : lo.x;
-            a2 = q ? lo.w : lo.y;
-            a1 = q ? hi.z : hi.x;
-            a3 = q ? hi.w : hi.y;
+            // piece s is this step's A fragment in register order (see the packed layout)
+            a0 = w[s].x;
+            a1 = w[s].y;
+            a2 = w[s].z;
+            a3 = w[s].w;
         }
         mma_bf16(d[s & 3], a0, a1, a2, a3, b0, b1);
     }
@@ -414,11 +413,15 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
             w[j] = make_uint4(__byte_perm(lo.x, 0u, 0x3120u), __byte_perm(lo.y, 0u, 0x3120u),
                               __byte_perm(hi.x, 0u, 0x3120u), __byte_perm(hi.y, 0u, 0x3120u));
         } else {
-            // piece j: row g + 8 (j / kRuns), run t = j % kRuns
-            const int r = g + 8 * (j / kRuns), k = 32 * (j % kRuns) + 8 * c;
-            w[j] = (r < rows && k < klen)
-                       ? *reinterpret_cast<const uint4*>(tile + (static_cast<size_t>(r) * klen + k) * 2)
-                       : make_uint4(0u, 0u, 0u, 0u);
+            // piece j = k-step j's A fragment: 4 bf16 at k0 of rows g and g + 8, as pairs
+            const int k0 = 32 * (j >> 1) + 8 * c + 4 * (j & 1);
+            const uint2 lo = (g < rows && k0 < klen)
+                                 ? *reinterpret_cast<const uint2*>(tile + (static_cast<size_t>(g) * klen + k0) * 2)
+                                 : make_uint2(0u, 0u);
+            const uint2 hi = (g + 8 < rows && k0 < klen)
+                                 ? *reinterpret_cast<const uint2*>(tile + (static_cast<size_t>(g + 8) * klen + k0) * 2)
+                                 : make_uint2(0u, 0u);
+            w[j] = make_uint4(lo.x, hi.x, lo.y, hi.y);
         }
     }
     uint4 xv[kRuns];

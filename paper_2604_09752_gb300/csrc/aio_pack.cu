@@ -2,10 +2,11 @@
 //
 // Tiles are 16 rows x 256 k; consecutive tiles are contiguous, so any run of them is one bulk copy.
 // A full tile (16 rows, 256 k) is stored in the order the stream kernel's lanes read it: lane
-// L = 4 r + c (r = 0..7, c = 0..3) reads 16-byte piece j at byte j * 512 + 16 L of the tile, and
-// its pieces hold runs of 8 consecutive k, W[row][32 t + 8 c .. +8), t = 0..7:
-//   bf16: piece j = 8 h + t holds row r + 8 h, run t;
-//   int8: piece j = 4 h + u holds row r + 8 h, runs t = 2u (bytes 0-7) and t = 2u + 1 (bytes 8-15),
+// L = 4 r + c (r = 0..7, c = 0..3) reads 16-byte piece j at byte j * 512 + 16 L of the tile:
+//   bf16: piece s (0..15) is one MMA's A fragment for k-step s, k0 = 32 (s/2) + 8 c + 4 (s%2):
+//         words W[r][k0..k0+1], W[r+8][k0..k0+1], W[r][k0+2..k0+3], W[r+8][k0+2..k0+3];
+//   int8: pieces hold runs of 8 consecutive k, W[row][32 t + 8 c .. +8); piece j = 4 h + u holds
+//         row r + 8 h, runs t = 2u (bytes 0-7) and t = 2u + 1 (bytes 8-15),
 //         each 4-code word of a run stored as codes (0, 2, 1, 3): the first k pair in the low bytes
 //         of the word's 16-bit halves, the second in the high bytes (the swap is its own inverse).
 // Every 128-bit shared-memory load of a warp is then contiguous.  Ragged tiles (last row group or
@@ -34,21 +35,33 @@ __global__ void __launch_bounds__(256) aio_pack_kernel(const uint8_t* __restrict
         const int rows = min(kRows, N - g * kRows);
         const int klen = min(kKT, K - kt * kKT);
         const size_t tile = (static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT) * E;
-        size_t in_tile;
-        if (rows == kRows && klen == kKT) {
-            const int h = r >> 3, lane = (r & 7) * 4 + ((kk & 31) >> 3), t = kk >> 5;
-            if (E == 2) {
-                in_tile = static_cast<size_t>((kKT / 32) * h + t) * 512 + lane * 16 + (kk & 7) * 2;
+        const bool full = rows == kRows && klen == kKT;
+        const size_t rowmajor = (static_cast<size_t>(n) * K + k) * E;
+        if (E == 2 && full) {
+            // 4 bf16 at k0 = kk: pair (k0, k0+1) is word h of piece s, pair (k0+2, k0+3) word 2 + h
+            const int h = r >> 3, lane = (r & 7) * 4 + ((kk >> 3) & 3), s = 2 * (kk >> 5) + ((kk >> 2) & 1);
+            uint8_t* piece = (INVERSE ? const_cast<uint8_t*>(src) : dst) + tile + static_cast<size_t>(s) * 512 + lane * 16;
+            uint32_t* w0 = reinterpret_cast<uint32_t*>(piece) + h;
+            uint32_t* w1 = reinterpret_cast<uint32_t*>(piece) + 2 + h;
+            if (INVERSE) {
+                *reinterpret_cast<uint2*>(dst + rowmajor) = make_uint2(*w0, *w1);
             } else {
-                in_tile = static_cast<size_t>((kKT / 64) * h + (t >> 1)) * 512 + lane * 16 + (t & 1) * 8;
+                const uint2 v = *reinterpret_cast<const uint2*>(src + rowmajor);
+                *w0 = v.x;
+                *w1 = v.y;
             }
+            continue;
+        }
+        size_t in_tile;
+        if (full) {
+            const int h = r >> 3, lane = (r & 7) * 4 + ((kk & 31) >> 3), t = kk >> 5;
+            in_tile = static_cast<size_t>((kKT / 64) * h + (t >> 1)) * 512 + lane * 16 + (t & 1) * 8;
         } else {
             in_tile = (static_cast<size_t>(r) * klen + kk) * E;
         }
         const size_t packed = tile + in_tile;
-        const size_t rowmajor = (static_cast<size_t>(n) * K + k) * E;
         uint2 v = *reinterpret_cast<const uint2*>(src + (INVERSE ? packed : rowmajor));
-        if (E == 1 && rows == kRows && klen == kKT) {   // swap bytes 1 and 2 of each word
+        if (E == 1 && full) {   // swap bytes 1 and 2 of each word
             v.x = __byte_perm(v.x, 0u, 0x3120u);
             v.y = __byte_perm(v.y, 0u, 0x3120u);
         }

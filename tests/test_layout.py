@@ -61,16 +61,19 @@ def _pack_index(idx, esize):
 
 
 def test_full_tile_fragment_order_bf16():
-    # lane L = 4r + c reads piece j (16 B) at byte j*512 + 16L: row r + 8*(j // 8), k = 32*(j % 8) + 8c .. +8
+    # lane L = 4r + c reads piece s (16 B) at byte s*512 + 16L: one MMA A fragment for k-step s,
+    # k0 = 32*(s // 2) + 8c + 4*(s % 2): W[r, k0:k0+2], W[r+8, k0:k0+2], W[r, k0+2:k0+4], W[r+8, k0+2:k0+4]
     T = layout.K_TILE
     assert T == 256
     order = layout._full_tile_order(2)
     assert np.array_equal(np.sort(order), np.arange(16 * T))
-    cases = {(0, 0): (0, 0), (0, 1): (0, 8), (7, 3): (0, 32 * 7 + 24), (8, 0): (8, 0), (15, 31): (15, 224 + 24),
-             (3, 5): (1, 96 + 8), (9, 30): (7 + 8, 32 + 16)}
-    for (j, L), (row, k0) in cases.items():
-        pos = (j * 512 + L * 16) // 2
-        assert list(order[pos:pos + 8]) == [row * T + k0 + e for e in range(8)], (j, L)
+    cases = {(0, 0): (0, 0), (1, 0): (0, 4), (0, 1): (0, 8), (2, 0): (0, 32), (15, 31): (7, 224 + 24 + 4),
+             (5, 6): (1, 64 + 16 + 4), (8, 13): (3, 128 + 8)}
+    for (s, L), (r, k0) in cases.items():
+        pos = (s * 512 + L * 16) // 2
+        want = [(r, k0), (r, k0 + 1), (r + 8, k0), (r + 8, k0 + 1), (r, k0 + 2), (r, k0 + 3), (r + 8, k0 + 2),
+                (r + 8, k0 + 3)]
+        assert list(order[pos:pos + 8]) == [row * T + k for row, k in want], (s, L)
 
 
 def test_full_tile_fragment_order_int8():
