@@ -165,15 +165,36 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
+// The constants of the int8 -> bf16 conversion, held in registers: a hardware LOP3 takes at most
+// one immediate, so (t & mask) | magic with both as immediates would cost two instructions.  The
+// moves are volatile so the compiler keeps the values in registers.
+struct I8Consts {
+    uint32_t m7, m8, magic;   // 0x007F007F, 0x00800080, 0x43004300
+};
+
+__device__ __forceinline__ I8Consts i8_consts() {
+    I8Consts k;
+    asm volatile("mov.u32 %0, 0x007F007F;" : "=r"(k.m7));
+    asm volatile("mov.u32 %0, 0x00800080;" : "=r"(k.m8));
+    asm volatile("mov.u32 %0, 0x43004300;" : "=r"(k.magic));
+    return k;
+}
+
+__device__ __forceinline__ uint32_t lop3_and_or(uint32_t t, uint32_t m, uint32_t c) {   // (t & m) | c
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(t), "r"(m), "r"(c));
+    return r;
+}
+
 // Two int8 codes -> bf16x2, exactly.  t holds the codes in the low bytes of its 16-bit halves (the
 // high bytes are ignored): 0x4300 | (q & 0x7F) is bf16 128 + (q & 0x7F), and 0x4300 | (q & 0x80)
-// is bf16 128 or 256; their difference is q.
-__device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t t) {
-    const uint32_t a = (t & 0x007F007Fu) | 0x43004300u;
-    const uint32_t b = (t & 0x00800080u) | 0x43004300u;
-    __nv_bfloat162 r = __hsub2(*reinterpret_cast<const __nv_bfloat162*>(&a),
-                               *reinterpret_cast<const __nv_bfloat162*>(&b));
-    return *reinterpret_cast<uint32_t*>(&r);
+// is bf16 128 or 256; their difference is q (an integer in [-128, 127], so the subtraction is exact).
+__device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t t, const I8Consts& k) {
+    const uint32_t a = lop3_and_or(t, k.m7, k.magic);
+    const uint32_t b = lop3_and_or(t, k.m8, k.magic);
+    uint32_t r;
+    asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
 }
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
@@ -356,7 +377,7 @@ constexpr int kRuns = kKT / 32;   // runs of 8 k per lane and row: x pieces per 
 
 template <bool I8>
 __device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)[TileT<I8>::kPieces],
-                                              const uint4 (&xv)[kRuns]) {
+                                              const uint4 (&xv)[kRuns], const I8Consts& kc) {
 #pragma unroll
     for (int s = 0; s < kKT / 16; ++s) {
         const int t = s >> 1, q = s & 1;
@@ -372,10 +393,10 @@ __device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)
             const int wi = (t & 1) * 2 + q;
             const uint32_t wl = wi == 0 ? lo.x : wi == 1 ? lo.y : wi == 2 ? lo.z : lo.w;
             const uint32_t wh = wi == 0 ? hi.x : wi == 1 ? hi.y : wi == 2 ? hi.z : hi.w;
-            a0 = i8x2_to_bf16x2(wl);
-            a2 = i8x2_to_bf16x2(wl >> 8);
-            a1 = i8x2_to_bf16x2(wh);
-            a3 = i8x2_to_bf16x2(wh >> 8);
+            a0 = i8x2_to_bf16x2(wl, kc);
+            a2 = i8x2_to_bf16x2(wl >> 8, kc);
+            a1 = i8x2_to_bf16x2(wh, kc);
+            a3 = i8x2_to_bf16x2(wh >> 8, kc);
         } else {
             // piece s is this step's A fragment in register order (see the packed layout)
             a0 = w[s].x;
@@ -393,7 +414,7 @@ __device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)
 // x is read from xp = x + token g's row (row stride xstride elements), staged or global.
 template <bool I8>
 __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, int rows, int klen, int kbase,
-                                         int lane, const Proj& P, const uint16_t* xrow_ptr) {
+                                         int lane, const Proj& P, const uint16_t* xrow_ptr, const I8Consts& kc) {
     using TL = TileT<I8>;
     constexpr int NP = TL::kPieces;
     const int g = lane >> 2, c = lane & 3;
@@ -431,14 +452,15 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
         const int k = 32 * t + 8 * c;
         xv[t] = (xrow && k < klen) ? *reinterpret_cast<const uint4*>(xrow_ptr + kbase + k) : make_uint4(0u, 0u, 0u, 0u);
     }
-    tile_mma_frag<I8>(d, w, xv);
+    tile_mma_frag<I8>(d, w, xv, kc);
 }
 
 // A full packed tile with x in global memory: xp = x + token min(g, M-1)'s row + 256 kt + 8c.
 // Lanes g >= M load a real token's x (the same addresses as lanes of token M-1, served once):
 // they only fill columns of D for tokens >= M, which are never written.  No select is needed.
 template <bool I8>
-__device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp) {
+__device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp,
+                                              const I8Consts& kc) {
     using TL = TileT<I8>;
     uint4 w[TL::kPieces];
 #pragma unroll
@@ -446,7 +468,7 @@ __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* t
     uint4 xv[kRuns];
 #pragma unroll
     for (int t = 0; t < kRuns; ++t) xv[t] = *reinterpret_cast<const uint4*>(xp + 32 * t);
-    tile_mma_frag<I8>(d, w, xv);
+    tile_mma_frag<I8>(d, w, xv, kc);
 }
 
 // A full packed tile with x staged in shared memory: waddr / xaddr are shared-window addresses of
@@ -455,7 +477,7 @@ __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* t
 // same addresses as token M-1's lanes (a broadcast), so the x loads are free of bank conflicts and
 // need no select; those lanes only fill columns of D for tokens >= M, which are never written.
 template <bool I8>
-__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr) {
+__device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xaddr, const I8Consts& kc) {
     using TL = TileT<I8>;
     uint4 w[TL::kPieces];
 #pragma unroll
@@ -463,7 +485,7 @@ __device__ __forceinline__ void tile_mma_full_s(float (&d)[4][4], uint32_t waddr
     uint4 xv[kRuns];
 #pragma unroll
     for (int t = 0; t < kRuns; ++t) xv[t] = lds128(xaddr + 64 * t);
-    tile_mma_frag<I8>(d, w, xv);
+    tile_mma_frag<I8>(d, w, xv, kc);
 }
 
 template <bool I8>
@@ -652,6 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     }
     __syncthreads();   // the only CTA-wide barrier: barriers and sync words are initialised
     const uint64_t pol = policy_evict_first();
+    const I8Consts kc = i8_consts();
 
     // The issue cursor walks this warp's tiles of all projections in consumption order.
     ChunkCursor ring_cur;
@@ -755,11 +778,11 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                     if (j < nt) {
                         const int klen = kt == NKT - 1 ? last_len : kKT;
                         if (P.uniform && stage) {
-                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2));
+                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), kc);
                         } else if (P.uniform) {
-                            tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT);
+                            tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, kc);
                         } else {
-                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr);
+                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr, kc);
                         }
                         tp += rows * klen * E;
                         if (kt == NKT - 1 || t == tend - 1) {
