@@ -63,7 +63,10 @@ def kernel_source_hash():
 
 
 def committed_traffic(workload_name, launches_per_step):
-    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current kernel."""
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current kernel.
+
+    profiles/gemv_traffic.txt holds `kernel_src_sha <hash>` and one `dram_bytes_per_step.<workload>
+    <bytes>` line per captured workload (read + write bytes of one whole-step launch)."""
     p = os.path.join(ROOT, "profiles", "gemv_traffic.txt")
     if not os.path.exists(p):
         return None, "no committed ncu traffic summary"
@@ -75,9 +78,10 @@ def committed_traffic(workload_name, launches_per_step):
             kv[k] = v
     if kv.get("kernel_src_sha") != kernel_source_hash():
         return None, "kernel changed since the committed ncu capture"
-    if kv.get("workload") != workload_name or "dram_bytes_per_step" not in kv:
-        return None, f"committed capture is for workload {kv.get('workload')}"
-    return float(kv["dram_bytes_per_step"]) / launches_per_step, kv.get("note", "ncu dram__bytes_read+write")
+    key = "dram_bytes_per_step." + workload_name
+    if key not in kv:
+        return None, f"no committed ncu capture for workload {workload_name}"
+    return float(kv[key]) / launches_per_step, kv.get("note", "ncu dram__bytes_read.sum + dram__bytes_write.sum")
 
 
 class ClockSampler:
