@@ -1,4 +1,8 @@
-"""Build libaio.so (sm_103a) in-tree with nvcc: one object per .cu, compiled in parallel."""
+"""Build libaio.so (sm_103a) in-tree with nvcc: one object per .cu, compiled in parallel.
+
+AIO_DEFINES in the environment (space-separated NAME=VALUE) adds -D options, e.g.
+AIO_DEFINES="AIO_FFMA=1" builds the CUDA-core (FFMA) consumer instead of the tensor-core one.  The
+defines of the last build are recorded beside the library, and a change forces a rebuild."""
 from __future__ import annotations
 
 import concurrent.futures as cf
@@ -12,6 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libaio.so")
+STAMP = os.path.join(HERE, "_build", "defines.txt")
 SOURCES = ["aio_gemv.cu", "aio_pack.cu", "aio_api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -26,10 +31,14 @@ def _deps():
     return max(os.path.getmtime(f) for f in files)
 
 
+def _defines():
+    return sorted(os.environ.get("AIO_DEFINES", "").split())
+
+
 def _compile(src: str, verbose: bool) -> str:
     obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".o")
     cmd = [nvcc(), *ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "-I", INCLUDE, "-I", CSRC,
-           "-c", os.path.join(CSRC, src), "-o", obj]
+           *["-D" + d for d in _defines()], "-c", os.path.join(CSRC, src), "-o", obj]
     if verbose:
         cmd.insert(1, "-Xptxas=-v")
     r = subprocess.run(cmd, capture_output=True, text=True)
@@ -41,7 +50,9 @@ def _compile(src: str, verbose: bool) -> str:
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= _deps():
+    stamp = " ".join(_defines())
+    same = os.path.exists(STAMP) and open(STAMP).read() == stamp
+    if not force and same and os.path.exists(LIB) and os.path.getmtime(LIB) >= _deps():
         return LIB
     os.makedirs(BUILD_DIR, exist_ok=True)
     with cf.ThreadPoolExecutor(len(SOURCES)) as ex:
@@ -50,6 +61,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+    with open(STAMP, "w") as f:
+        f.write(stamp)
     return LIB
 
 

@@ -156,7 +156,7 @@ __device__ __forceinline__ unsigned atom_add_acq_rel_cta_shared(unsigned* p, uns
 }
 
 // D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
-__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+[[maybe_unused]] __device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                          uint32_t b0, uint32_t b1) {
     asm volatile(
         "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
@@ -189,7 +189,7 @@ __device__ __forceinline__ uint32_t lop3_and_or(uint32_t t, uint32_t m, uint32_t
 // Two int8 codes -> bf16x2, exactly.  t holds the codes in the low bytes of its 16-bit halves (the
 // high bytes are ignored): 0x4300 | (q & 0x7F) is bf16 128 + (q & 0x7F), and 0x4300 | (q & 0x80)
 // is bf16 128 or 256; their difference is q (an integer in [-128, 127], so the subtraction is exact).
-__device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t t, const I8Consts& k) {
+[[maybe_unused]] __device__ __forceinline__ uint32_t i8x2_to_bf16x2(uint32_t t, const I8Consts& k) {
     const uint32_t a = lop3_and_or(t, k.m7, k.magic);
     const uint32_t b = lop3_and_or(t, k.m8, k.magic);
     uint32_t r;
@@ -408,13 +408,109 @@ __device__ __forceinline__ void tile_mma_frag(float (&d)[4][4], const uint4 (&w)
     }
 }
 
+#if AIO_FFMA
+// ------------------------------------------------------------------ CUDA-core consumer (comparison)
+// Built with AIO_DEFINES="AIO_FFMA=1".  Same layouts, ring, partition and fixups; only the tile
+// arithmetic differs: lane (g, c) converts its weights of rows g and g + 8 at its k (the k order of
+// the MMA path) to fp32 and accumulates acc(h, m) = sum W[row g + 8h][k] x[m][k] with FFMA for every
+// token m, in d[(8h + m) / 4][(8h + m) % 4].  ffma_finish reduces over the four lanes of a row pair
+// and returns the D layout of the MMA path.
+__device__ __forceinline__ float& acc_at(float (&d)[4][4], int h, int m) { return d[(8 * h + m) >> 2][(8 * h + m) & 3]; }
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+// int8 code in byte i of u (u = stored word ^ 0x80808080) -> float, exactly: 2^23 + q + 128 - (2^23 + 128)
+__device__ __forceinline__ float i8f(uint32_t u, uint32_t i) {
+    return __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7440u | i)) - 8388736.0f;
+}
+__device__ __forceinline__ uint32_t word_of(const uint4& v, int i) { return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w; }
+
+template <bool I8, int MT, class XL>
+__device__ __forceinline__ void tile_ffma(float (&d)[4][4], const uint4 (&w)[TileT<I8>::kPieces], XL xload) {
+#pragma unroll
+    for (int t = 0; t < kRuns; ++t) {
+        uint4 xq[MT];
+#pragma unroll
+        for (int m = 0; m < MT; ++m) xq[m] = xload(m, t);
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            float wg[4], wh[4];   // k0 .. k0 + 3 of rows g and g + 8
+            if constexpr (I8) {
+                const int wi = (t & 1) * 2 + q;   // stored (0, 2, 1, 3)
+                const uint32_t a = word_of(w[t >> 1], wi) ^ 0x80808080u;
+                const uint32_t b = word_of(w[kRuns / 2 + (t >> 1)], wi) ^ 0x80808080u;
+                wg[0] = i8f(a, 0); wg[1] = i8f(a, 2); wg[2] = i8f(a, 1); wg[3] = i8f(a, 3);
+                wh[0] = i8f(b, 0); wh[1] = i8f(b, 2); wh[2] = i8f(b, 1); wh[3] = i8f(b, 3);
+            } else {
+                const uint4& a = w[2 * t + q];
+                wg[0] = bf_lo(a.x); wg[1] = bf_hi(a.x); wg[2] = bf_lo(a.z); wg[3] = bf_hi(a.z);
+                wh[0] = bf_lo(a.y); wh[1] = bf_hi(a.y); wh[2] = bf_lo(a.w); wh[3] = bf_hi(a.w);
+            }
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+                const uint32_t xa = q ? xq[m].z : xq[m].x, xb = q ? xq[m].w : xq[m].y;
+                const float x0 = bf_lo(xa), x1 = bf_hi(xa), x2 = bf_lo(xb), x3 = bf_hi(xb);
+                float& a0 = acc_at(d, 0, m);
+                float& a1 = acc_at(d, 1, m);
+                a0 = fmaf(wg[3], x3, fmaf(wg[2], x2, fmaf(wg[1], x1, fmaf(wg[0], x0, a0))));
+                a1 = fmaf(wh[3], x3, fmaf(wh[2], x2, fmaf(wh[1], x1, fmaf(wh[0], x0, a1))));
+            }
+        }
+    }
+}
+
+// Group end: sum over the lanes c of each row pair, then lane (g, c) returns D[g][2c], D[g][2c+1],
+// D[g+8][2c], D[g+8][2c+1] (0 for tokens >= M), as the MMA path does.
+template <int MT>
+__device__ __forceinline__ void ffma_finish(float (&d)[4][4], float (&sum)[4], int lane) {
+    float r0[8], r1[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+        float a = m < MT ? acc_at(d, 0, m) : 0.0f, b = m < MT ? acc_at(d, 1, m) : 0.0f;
+        if (m < MT) {
+            a += __shfl_xor_sync(0xffffffffu, a, 1);
+            a += __shfl_xor_sync(0xffffffffu, a, 2);
+            b += __shfl_xor_sync(0xffffffffu, b, 1);
+            b += __shfl_xor_sync(0xffffffffu, b, 2);
+        }
+        r0[m] = a;
+        r1[m] = b;
+    }
+    const int c = lane & 3;
+    sum[0] = c == 0 ? r0[0] : c == 1 ? r0[2] : c == 2 ? r0[4] : r0[6];
+    sum[1] = c == 0 ? r0[1] : c == 1 ? r0[3] : c == 2 ? r0[5] : r0[7];
+    sum[2] = c == 0 ? r1[0] : c == 1 ? r1[2] : c == 2 ? r1[4] : r1[6];
+    sum[3] = c == 0 ? r1[1] : c == 1 ? r1[3] : c == 2 ? r1[5] : r1[7];
+}
+
+// Full tile, x staged: xs0 = shared address of token 0's x at k = 256 kt + 8c, xsb = row stride in bytes.
+template <bool I8, int MT>
+__device__ __forceinline__ void ffma_full_s(float (&d)[4][4], uint32_t waddr, uint32_t xs0, uint32_t xsb) {
+    uint4 w[TileT<I8>::kPieces];
+#pragma unroll
+    for (int j = 0; j < TileT<I8>::kPieces; ++j) w[j] = lds128(waddr + j * 512);
+    tile_ffma<I8, MT>(d, w, [&](int m, int t) { return lds128(xs0 + m * xsb + 64 * t); });
+}
+
+// Full tile, x in global memory: x0 = x + 256 kt + 8c (token 0), K = row stride.
+template <bool I8, int MT>
+__device__ __forceinline__ void ffma_full_g(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* x0, int K) {
+    uint4 w[TileT<I8>::kPieces];
+#pragma unroll
+    for (int j = 0; j < TileT<I8>::kPieces; ++j) w[j] = *reinterpret_cast<const uint4*>(tile_lane + j * 512);
+    tile_ffma<I8, MT>(d, w, [&](int m, int t) {
+        return *reinterpret_cast<const uint4*>(x0 + static_cast<size_t>(m) * K + 32 * t);
+    });
+}
+#endif  // AIO_FFMA
+
 // Any tile: full packed tiles in fragment order (piece j at j * 512 + 16 lane); ragged tiles
 // (rows < 16 or klen < 256) and row-major weights as the row-major block [rows][klen].  Pieces
 // outside the tile are zero, and so is x outside [kbase, kbase + klen) or for tokens >= M.
 // x is read from xp = x + token g's row (row stride xstride elements), staged or global.
 template <bool I8>
 __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, int rows, int klen, int kbase,
-                                         int lane, const Proj& P, const uint16_t* xrow_ptr, const I8Consts& kc) {
+                                         int lane, const Proj& P, const uint16_t* xrow_ptr, const I8Consts& kc,
+                                         int xstride = 0) {
     using TL = TileT<I8>;
     constexpr int NP = TL::kPieces;
     const int g = lane >> 2, c = lane & 3;
@@ -445,6 +541,14 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
             w[j] = make_uint4(lo.x, hi.x, lo.y, hi.y);
         }
     }
+#if AIO_FFMA
+    // xrow_ptr is token 0's row here, xstride the row stride (staged or global)
+    tile_ffma<I8, kMaxM>(d, w, [&](int m, int t) {
+        const int k = 32 * t + 8 * c;
+        return (m < P.M && k < klen) ? *reinterpret_cast<const uint4*>(xrow_ptr + static_cast<size_t>(m) * xstride + kbase + k)
+                                     : make_uint4(0u, 0u, 0u, 0u);
+    });
+#else
     uint4 xv[kRuns];
     const bool xrow = g < P.M;
 #pragma unroll
@@ -453,6 +557,7 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
         xv[t] = (xrow && k < klen) ? *reinterpret_cast<const uint4*>(xrow_ptr + kbase + k) : make_uint4(0u, 0u, 0u, 0u);
     }
     tile_mma_frag<I8>(d, w, xv, kc);
+#endif
 }
 
 // A full packed tile with x in global memory: xp = x + token min(g, M-1)'s row + 256 kt + 8c.
@@ -761,9 +866,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             int rows = min(kRows, P.N - g * kRows);
             const int tok = lane >> 2;
             // x of this lane's token (rows >= M are never read): the staged copy or global memory
-            const uint16_t* xrow_ptr = stage ? xs + tok * xs_stride : P.x + static_cast<size_t>(tok) * P.K;
+            [[maybe_unused]] const uint16_t* xrow_ptr = stage ? xs + tok * xs_stride : P.x + static_cast<size_t>(tok) * P.K;
             const int xtok = min(tok, MT - 1);   // full tiles: lanes of tokens >= M read token M-1's x
-            const uint16_t* xlane = P.x + static_cast<size_t>(xtok) * P.K + 8 * (lane & 3);
+            [[maybe_unused]] const uint16_t* xlane = P.x + static_cast<size_t>(xtok) * P.K + 8 * (lane & 3);
             const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>((xtok * xs_stride + 8 * (lane & 3)) * 2);
             while (t < tend) {
                 if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
@@ -777,6 +882,17 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 for (int j = 0; j < C; ++j) {
                     if (j < nt) {
                         const int klen = kt == NKT - 1 ? last_len : kKT;
+#if AIO_FFMA
+                        if (P.uniform && stage) {
+                            ffma_full_s<I8, MT>(d, smem_addr(tp) + lane * 16,
+                                                smem_addr(xs) + 16 * (lane & 3) + kt * (kKT * 2), xs_stride * 2);
+                        } else if (P.uniform) {
+                            ffma_full_g<I8, MT>(d, tp + lane * 16, P.x + 8 * (lane & 3) + kt * kKT, P.K);
+                        } else {
+                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, stage ? xs : P.x, kc,
+                                         stage ? xs_stride : P.K);
+                        }
+#else
                         if (P.uniform && stage) {
                             tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), kc);
                         } else if (P.uniform) {
@@ -784,11 +900,16 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                         } else {
                             tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr, kc);
                         }
+#endif
                         tp += rows * klen * E;
                         if (kt == NKT - 1 || t == tend - 1) {
                             float sum[4];
+#if AIO_FFMA
+                            ffma_finish<MT>(d, sum, lane);
+#else
 #pragma unroll
                             for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
+#endif
                             if (!finish_group<I8>(P, s, Z, sum, g, rows, z, t0, t1, lane)) {
                                 if (lane == 0) atomicCAS(s.err, 0, kDevErrTimeout);
                                 dead = true;

@@ -11,6 +11,9 @@
 #ifndef AIO_WARPS
 #define AIO_WARPS 8             // warps per CTA (one CTA per SM)
 #endif
+#ifndef AIO_FFMA
+#define AIO_FFMA 0              // 1: CUDA-core FFMA consumer instead of mma.sync (kept for comparison)
+#endif
 #ifndef AIO_SLOT_KB
 #define AIO_SLOT_KB 8           // bytes per ring slot, KB: one bulk copy of consecutive tiles
 #endif
