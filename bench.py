@@ -418,12 +418,55 @@ def run_ours(args, wl):
             "clocks": clk,
             "setup_s": round(setup_s, 1),
             "cpu_baseline": cpu,
+            # The paper's own decode rates on Ascend 910B, FP16 at 2K context (Tab. 3, Tab. 4): context only.
+            "paper_context": {"hardware": "Ascend 910B", "tokens_per_s_1b": 21.58, "tokens_per_s_7b": 17.18,
+                              "tokens_per_s_a_io_scenario_a": 19.80},
         }
         print(json.dumps(line), flush=True)
     dw.close()
+    if args.pld_sweep and rank == 0:
+        pld_sweep(args, peak)
     if pg is not None:
         pg.destroy_process_group()
     return 0
+
+
+def pld_sweep(args, peak):
+    """Prompt-lookup verification widths (Sec. 4.2): the 7B-class step at M = 1, 2, 4, 8 for bf16 and
+    int8 weights, one weight set per type, one JSON line per (type, M) after the main line."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    from synth import workloads as swl
+    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
+    for wt in ("bf16", "int8"):
+        wl = swl.pld_workload(8, wt)
+        dw = DeviceWorkload(wl, seed=args.seed, max_M=8)
+        wbytes = dw.weight_bytes()
+        stream = torch.cuda.Stream()
+        for M in swl.PLD_WIDTHS:
+            dw.fill_x(M)
+            step = dw.step_handle(M, flags)
+            with torch.cuda.stream(stream):
+                for _ in range(args.warmup):
+                    aio.aio_decode_step(step, stream.cuda_stream)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(args.steps):
+                aio.aio_decode_step(step, stream.cuda_stream)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            assert aio.aio_decode_step_check(step) == 0
+            ms = e0.elapsed_time(e1) / args.steps
+            gbs = wbytes / (ms / 1e3) / 1e9
+            print(json.dumps({"sweep": "pld", "workload": f"7b-pld-{wt}-M{M}", "M": M, "wtype": wt,
+                              "ms_per_step": round(ms, 4), "value": round(gbs, 2), "unit": "GB/s",
+                              "frac_of_measured_peak": round(gbs / peak, 4),
+                              "tokens_per_s": round(1000.0 / ms, 2),
+                              "verified_tokens_per_s_upper_bound": round(1000.0 * M / ms, 2),
+                              "steps": args.steps, "warmup": args.warmup}), flush=True)
+        dw.close()
 
 
 def main():
@@ -438,6 +481,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="repeat oracle passes over the row sample for at least this long")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--pld-sweep", action="store_true",
+                    help="after the main line, one line per PLD width M in {1,2,4,8} for bf16 and int8 7B steps")
     ap.add_argument("--step-mode", choices=["persistent", "chain"], default="persistent",
                     help="one cooperative launch per step (default) or one launch per projection")
     args = ap.parse_args()
