@@ -203,7 +203,9 @@ template <bool I8>
 struct TileT {
     static constexpr int kEsize = I8 ? 1 : 2;
     static constexpr int kBytes = kRows * kKT * kEsize;    // 4096 (int8) or 8192 (bf16)
-    static constexpr int kChunk = kSlotBytes / kBytes;     // tiles per ring slot
+    static constexpr int kSlot = I8 ? kSlotBytesI8 : kSlotBytes;
+    static constexpr int kStagesT = I8 ? kStagesI8 : kStages;   // ring slots per warp
+    static constexpr int kChunk = kSlot / kBytes;          // tiles per ring slot
     static constexpr int kPieces = kBytes / 512;           // 16-byte pieces per lane per tile (8 or 16)
 };
 
@@ -603,6 +605,7 @@ __device__ __forceinline__ float row_scale(const Proj& P, int n) {
 }
 
 constexpr uint32_t kSlotEmpty = 0xFFFFFFFFu;   // a partial slot not written yet
+constexpr int kGather = 8;                    // contributors whose slots an owner loads at once
 
 // A partial sum as stored in a slot: NaNs become the quiet NaN 0x7FC00000, so no stored value is
 // ever kSlotEmpty.
@@ -615,7 +618,7 @@ __device__ __forceinline__ uint32_t slot_bits(float v) {
 // complete in this warp), stores the partial (split group, not the owner), or, as the owner, adds
 // the other contributors' partials and writes y.  Returns false if a wait for a partial expired or
 // the launch already failed.
-template <bool I8>
+template <bool I8, int MT>
 __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s, int Z, const float (&d)[4], int g,
                                              int rows, long long z, long long t0, long long t1, int lane) {
     const int gr = lane >> 2, m0 = 2 * (lane & 3);
@@ -632,7 +635,7 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
         return true;
     }
 
-    const int V = kRows * P.M;
+    constexpr int V = kRows * MT;   // values per partial slot (P.M == MT)
     if (t0 > gfirst) {
         // Not the owner: g is this warp's first group (its last split group it always owns), so
         // one slot per warp suffices.  Publish [token][row] and go on.
@@ -646,49 +649,95 @@ __device__ __forceinline__ bool finish_group(const Proj& P, const StreamArgs& s,
     }
 
     // The owner: this warp holds tile gfirst.  The other contributors are the next warps up to the
-    // owner of tile tl (segments are contiguous and in warp order).
+    // owner of tile tl (segments are contiguous and in warp order).  Lane l handles the values
+    // v = 32 j + l (token v / 16, row v % 16) for j < NV.
     long long zl = z;
     while (zl + 1 < Z && seg(static_cast<int>(zl) + 1, Z, P.Tq, P.Tr) <= tl) ++zl;
-    bool ok = true;
-    for (int v0 = 0; v0 < V; v0 += 32) {
-        const int v = v0 + lane;
+    constexpr int NV = (kRows * MT + 31) / 32;
+    float sum[NV];
+    bool act[NV];
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+        const int v = 32 * j + lane;
         const int m = v / kRows, r = v - m * kRows;
         const int src = ((r & 7) * 4 + (m >> 1)) & 31;   // the lane holding the owner's own value
         const int idx = (r >> 3) * 2 + (m & 1);
         const float o0 = __shfl_sync(0xffffffffu, d[0], src), o1 = __shfl_sync(0xffffffffu, d[1], src);
         const float o2 = __shfl_sync(0xffffffffu, d[2], src), o3 = __shfl_sync(0xffffffffu, d[3], src);
-        if (v < V && r < rows) {
-            float sum = idx == 0 ? o0 : idx == 1 ? o1 : idx == 2 ? o2 : o3;
-            // Four contributors at a time: their slots are loaded together (independent loads, one
-            // round trip), then added in warp order; only slots still empty are polled.
-            for (long long zb = z + 1; ok && zb <= zl; zb += 4) {
-                uint32_t bits[4];
+        act[j] = v < V && r < rows;
+        sum[j] = idx == 0 ? o0 : idx == 1 ? o1 : idx == 2 ? o2 : o3;
+    }
+    bool ok = true;
+    // Up to kGather contributors at a time: all their slots are loaded together (independent loads,
+    // one round trip), the ones still empty are re-loaded together until every slot is written,
+    // and the values are added in warp order.
+    for (long long zb = z + 1; ok && zb <= zl; zb += kGather) {
+        unsigned want = 0u;   // contributors with a non-empty segment (the others publish nothing)
+        int sprev = seg(static_cast<int>(zb), Z, P.Tq, P.Tr);
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    bits[i] = zb + i <= zl ? ld_relaxed_u32(P.partial + static_cast<size_t>(zb + i) * V + v) : 0u;
+        for (int i = 0; i < kGather; ++i) {
+            if (zb + i <= zl) {
+                const int snext = seg(static_cast<int>(zb + i) + 1, Z, P.Tq, P.Tr);
+                if (snext > sprev) want |= 1u << i;
+                sprev = snext;
+            }
+        }
+        const uint32_t* slots = reinterpret_cast<const uint32_t*>(P.partial) + static_cast<size_t>(zb) * V + lane;
+        uint32_t bits[NV][kGather];
+        uint32_t pend = 0u;   // bit j * kGather + i: value j of contributor zb + i not written yet
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const long long zz = zb + i;
-                    if (!ok || zz > zl) break;
-                    if (seg(static_cast<int>(zz) + 1, Z, P.Tq, P.Tr) == seg(static_cast<int>(zz), Z, P.Tq, P.Tr))
-                        continue;   // empty segment
-                    float* slot = P.partial + static_cast<size_t>(zz) * V + v;
-                    if (bits[i] == kSlotEmpty) {
-                        const uint64_t start = globaltimer_ns();
-                        while (ok && (bits[i] = ld_relaxed_u32(slot)) == kSlotEmpty)
-                            ok = ld_relaxed_u32(s.err) == 0u && globaltimer_ns() - start <= s.wait_limit_ns;
+        for (int j = 0; j < NV; ++j) {
+#pragma unroll
+            for (int i = 0; i < kGather; ++i) {
+                bits[j][i] = 0u;
+                if (act[j] && (want >> i & 1u)) bits[j][i] = ld_relaxed_u32(slots + i * V + 32 * j);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < NV; ++j)
+#pragma unroll
+            for (int i = 0; i < kGather; ++i)
+                if (act[j] && (want >> i & 1u) && bits[j][i] == kSlotEmpty) pend |= 1u << (j * kGather + i);
+        if (pend) {
+            const uint64_t start = globaltimer_ns();
+            while (pend && ok) {
+                uint32_t still = 0u;
+#pragma unroll
+                for (int j = 0; j < NV; ++j) {
+#pragma unroll
+                    for (int i = 0; i < kGather; ++i) {
+                        if (pend >> (j * kGather + i) & 1u) {
+                            bits[j][i] = ld_relaxed_u32(slots + i * V + 32 * j);
+                            if (bits[j][i] == kSlotEmpty) still |= 1u << (j * kGather + i);
+                        }
                     }
-                    if (ok) {
-                        sum += __uint_as_float(bits[i]);
-                        st_relaxed_u32(slot, kSlotEmpty);
+                }
+                pend = still;
+                if (pend) ok = ld_relaxed_u32(s.err) == 0u && globaltimer_ns() - start <= s.wait_limit_ns;
+            }
+        }
+        if (ok) {
+#pragma unroll
+            for (int j = 0; j < NV; ++j) {
+#pragma unroll
+                for (int i = 0; i < kGather; ++i) {
+                    if (act[j] && (want >> i & 1u)) {
+                        sum[j] += __uint_as_float(bits[j][i]);
+                        st_relaxed_u32(P.partial + (static_cast<size_t>(zb + i) * V + 32 * j + lane), kSlotEmpty);
                     }
                 }
             }
-            if (ok) P.y[static_cast<size_t>(m) * P.N + row0 + r] = sum * row_scale<I8>(P, row0 + r);
         }
-        if (!__all_sync(0xffffffffu, ok)) return false;   // uniform: every lane reaches this point
     }
-    return true;
+    if (ok) {
+#pragma unroll
+        for (int j = 0; j < NV; ++j) {
+            const int v = 32 * j + lane;
+            const int m = v / kRows, r = v - m * kRows;
+            if (act[j]) P.y[static_cast<size_t>(m) * P.N + row0 + r] = sum[j] * row_scale<I8>(P, row0 + r);
+        }
+    }
+    return __all_sync(0xffffffffu, ok);
 }
 
 // Lane 0 polls until *counter >= target (bounded by limit_ns); the result is broadcast to the warp.
@@ -748,7 +797,7 @@ template <int MT, bool I8>
 __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_constant__ StreamArgs s) {
     using TL = TileT<I8>;
     constexpr int C = TL::kChunk;
-    constexpr int S = kStages;
+    constexpr int S = TL::kStagesT;
     constexpr int E = TL::kEsize;
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5;
@@ -791,7 +840,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         int ip, it, nt;
         if (!cursor_next(ring_cur, s, z, Z, C, ip, it, nt)) return false;
         if (lane == 0 && !(stall && first_issue))   // test hook: this slot's barrier never completes
-            issue_chunk<I8>(ring_cur.cur, it, nt, ring + islot * kSlotBytes, &bars[islot], pol);
+            issue_chunk<I8>(ring_cur.cur, it, nt, ring + islot * TL::kSlot, &bars[islot], pol);
         first_issue = false;
         islot = (islot + 1 == S) ? 0 : islot + 1;
         return true;
@@ -801,6 +850,21 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         if (!issue_next()) break;
         ++in_flight;
     }
+    // Chunks of projections after the one being consumed may take at most AIO_AHEAD slots; the
+    // rest of the ring is topped up when the next projection starts.
+    int ahead = 0;
+    auto refill = [&](int p) {
+        const bool later = ring_cur.p > p || ring_cur.t >= ring_cur.te;
+        if (later && ahead >= AIO_AHEAD) {
+            --in_flight;
+            return;
+        }
+        if (!issue_next()) {
+            --in_flight;
+        } else if (later) {
+            ++ahead;
+        }
+    };
 
     // With programmatic dependent launch, everything below (x, y, workspace) waits for the
     // previous grid on the stream.
@@ -856,6 +920,10 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             }
             xphase ^= 1u;
         }
+        ahead = 0;
+        if (!dead) {
+            while (in_flight < S && issue_next()) ++in_flight;
+        }
         if (!dead && t1 > t0) {
             float d[4][4] = {};
             const int NKT = P.NKT;
@@ -877,7 +945,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                     break;
                 }
                 const int nt = min(C, tend - t);
-                const uint8_t* tp = ring + cslot * kSlotBytes;
+                const uint8_t* tp = ring + cslot * TL::kSlot;
 #pragma unroll
                 for (int j = 0; j < C; ++j) {
                     if (j < nt) {
@@ -910,7 +978,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
 #pragma unroll
                             for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
 #endif
-                            if (!finish_group<I8>(P, s, Z, sum, g, rows, z, t0, t1, lane)) {
+                            if (!finish_group<I8, MT>(P, s, Z, sum, g, rows, z, t0, t1, lane)) {
                                 if (lane == 0) atomicCAS(s.err, 0, kDevErrTimeout);
                                 dead = true;
                             }
@@ -932,7 +1000,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 __syncwarp();
                 cslot = (cslot + 1 == S) ? 0 : cslot + 1;
                 cphase ^= (cslot == 0) ? 1u : 0u;
-                if (!issue_next()) --in_flight;
+                refill(p);
             }
             if (dead) {
                 // wait (bounded) for this warp's copies still in flight, then stop issuing

@@ -17,6 +17,12 @@
 #ifndef AIO_SLOT_KB
 #define AIO_SLOT_KB 8           // bytes per ring slot, KB: one bulk copy of consecutive tiles
 #endif
+#ifndef AIO_AHEAD
+#define AIO_AHEAD 2             // ring slots a warp may fill with later projections while consuming one
+#endif
+#ifndef AIO_SLOT_KB_I8
+#define AIO_SLOT_KB_I8 AIO_SLOT_KB   // the same for int8 weights (4 KB tiles)
+#endif
 
 namespace aio {
 
@@ -27,8 +33,11 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kRingBytesPerWarp = AIO_RING_KB * 1024;
 constexpr int kSlotBytes = AIO_SLOT_KB * 1024;
 constexpr int kStages = kRingBytesPerWarp / kSlotBytes;  // ring slots per warp
-constexpr int kMaxStages = kStages;
-static_assert(kSlotBytes % 4096 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
+constexpr int kSlotBytesI8 = AIO_SLOT_KB_I8 * 1024;
+constexpr int kStagesI8 = kRingBytesPerWarp / kSlotBytesI8;
+constexpr int kMaxStages = kStages > kStagesI8 ? kStages : kStagesI8;
+static_assert(kSlotBytes % 8192 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
+static_assert(kSlotBytesI8 % 4096 == 0 && kStagesI8 >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
 constexpr int kSyncOffset = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;  // CTA-level sync words
 constexpr int kXsOffset = kSyncOffset + 32;        // sync words (16 B), the x barrier (8 B), padding
 constexpr int kXsPad = 32;                         // elements between staged x rows beyond K (64 B)
