@@ -206,6 +206,8 @@ struct TileT {
     static constexpr int kSlot = I8 ? kSlotBytesI8 : kSlotBytes;
     static constexpr int kStagesT = I8 ? kStagesI8 : kStages;   // ring slots per warp
     static constexpr int kChunk = kSlot / kBytes;          // tiles per ring slot
+    static constexpr int kAhead = I8 ? AIO_AHEAD_I8 : AIO_AHEAD;
+    static constexpr int kAheadLive = I8 ? AIO_AHEAD_LIVE_I8 : AIO_AHEAD_LIVE;
     static constexpr int kPieces = kBytes / 512;           // 16-byte pieces per lane per tile (8 or 16)
 };
 
@@ -850,12 +852,13 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         if (!issue_next()) break;
         ++in_flight;
     }
-    // Chunks of projections after the one being consumed may take at most AIO_AHEAD slots; the
-    // rest of the ring is topped up when the next projection starts.
+    // Chunks of projections after the one being consumed take at most TL::kAheadLive slots while
+    // the warp still has tiles of the current one, TL::kAhead once it has finished them (its last
+    // gather done); the rest of the ring is filled when the next projection starts.
     int ahead = 0;
     auto refill = [&](int p) {
         const bool later = ring_cur.p > p || ring_cur.t >= ring_cur.te;
-        if (later && ahead >= AIO_AHEAD) {
+        if (later && ahead >= TL::kAheadLive) {
             --in_flight;
             return;
         }
@@ -1001,6 +1004,12 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 cslot = (cslot + 1 == S) ? 0 : cslot + 1;
                 cphase ^= (cslot == 0) ? 1u : 0u;
                 refill(p);
+            }
+            if (!dead) {
+                while (ahead < TL::kAhead && in_flight < S && issue_next()) {
+                    ++in_flight;
+                    ++ahead;
+                }
             }
             if (dead) {
                 // wait (bounded) for this warp's copies still in flight, then stop issuing

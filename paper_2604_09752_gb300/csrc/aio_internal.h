@@ -17,8 +17,20 @@
 #ifndef AIO_SLOT_KB
 #define AIO_SLOT_KB 8           // bytes per ring slot, KB: one bulk copy of consecutive tiles
 #endif
+// Ring slots a warp fills with chunks of the next projection once it has finished its tiles of the
+// current one (AIO_AHEAD), and while it still has some (AIO_AHEAD_LIVE); the rest of the ring is
+// filled when the next projection starts.  Separate values for int8 weights.
 #ifndef AIO_AHEAD
-#define AIO_AHEAD 2             // ring slots a warp may fill with later projections while consuming one
+#define AIO_AHEAD 2
+#endif
+#ifndef AIO_AHEAD_LIVE
+#define AIO_AHEAD_LIVE 0
+#endif
+#ifndef AIO_AHEAD_I8
+#define AIO_AHEAD_I8 2
+#endif
+#ifndef AIO_AHEAD_LIVE_I8
+#define AIO_AHEAD_LIVE_I8 2
 #endif
 #ifndef AIO_SLOT_KB_I8
 #define AIO_SLOT_KB_I8 AIO_SLOT_KB   // the same for int8 weights (4 KB tiles)
