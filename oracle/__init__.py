@@ -16,10 +16,22 @@ Functions and the passages they follow:
   * bf16_to_double(h)        decoding of a bf16 bit pattern.
   * pack_tiles / unpack_tiles  the tiled weight layout the CUDA packer must
                              produce (a pure permutation; see layout.py).
+  * double_to_bf16(v)        round a double to bf16, nearest-even.
+  * silu(t), rmsnorm(...), swiglu(...), slice_x(...)
+                             the steps between the projections of a chained
+                             decoder step; chain_step(...) runs a whole chained
+                             step.  The paper prints no block structure (it
+                             names its models, Sec. 4.2): the reading is a
+                             pre-norm decoder block (RMSNorm, attention, SwiGLU
+                             MLP, residual adds) whose attention covers one
+                             position, so it returns the V third of QKV.
 
 Parity status: every function above is pinned by tests/test_oracle_pins.py
 (brute force, one-hot, identity/zero, linearity, exact dequant, fp64 error
-bound against exact rational sums) and tests/test_oracle_mutants.py.
+bound against exact rational sums), tests/test_oracle_chain_pins.py (bf16
+rounding against exact rationals and a library conversion, closed forms of the
+logistic, RMSNorm invariants, exact residual adds) and
+tests/test_oracle_mutants.py.
 """
 from __future__ import annotations
 
@@ -48,6 +60,16 @@ def load(path: str = LIB_PATH):
     lib.aio_oracle_linear_i8.argtypes = [vp, vp, vp, i64, i64, i64, vp]
     lib.aio_oracle_dequant_i8.restype = None
     lib.aio_oracle_dequant_i8.argtypes = [vp, vp, i64, i64, vp]
+    lib.aio_oracle_double_to_bf16.restype = ctypes.c_uint16
+    lib.aio_oracle_double_to_bf16.argtypes = [ctypes.c_double]
+    lib.aio_oracle_silu.restype = ctypes.c_double
+    lib.aio_oracle_silu.argtypes = [ctypes.c_double]
+    lib.aio_oracle_rmsnorm.restype = None
+    lib.aio_oracle_rmsnorm.argtypes = [vp, vp, vp, i64, i64, ctypes.c_double, vp, vp]
+    lib.aio_oracle_swiglu.restype = None
+    lib.aio_oracle_swiglu.argtypes = [vp, i64, i64, i64, vp]
+    lib.aio_oracle_slice.restype = None
+    lib.aio_oracle_slice.argtypes = [vp, i64, i64, i64, i64, vp]
     return lib
 
 
@@ -109,6 +131,75 @@ class Oracle:
         self.lib.aio_oracle_dequant_i8(q.ctypes.data, s.ctypes.data, N, K, Wd.ctypes.data)
         return Wd
 
+    def double_to_bf16(self, v) -> int:
+        return int(self.lib.aio_oracle_double_to_bf16(float(v)))
+
+    def silu(self, t) -> float:
+        return float(self.lib.aio_oracle_silu(float(t)))
+
+    def rmsnorm(self, h_in, r, gamma, eps):
+        """(h_out, x): h_out = fp32(h_in + r) (r may be None), x = bf16(h_out * gamma / rms(h_out))."""
+        h_in = _c(h_in, np.float32)
+        M, K = h_in.shape
+        rr = None if r is None else _c(r, np.float32).reshape(M, K)
+        g = _c(gamma, np.uint16)
+        assert g.shape == (K,)
+        h_out = np.empty((M, K), np.float32)
+        x = np.empty((M, K), np.uint16)
+        self.lib.aio_oracle_rmsnorm(h_in.ctypes.data, None if rr is None else rr.ctypes.data, g.ctypes.data, M, K,
+                                    float(eps), h_out.ctypes.data, x.ctypes.data)
+        return h_out, x
+
+    def swiglu(self, y, I):
+        """x[m, k] = bf16(silu(y[m, k]) * y[m, I + k]) for k < I; y [M, stride >= 2I] fp32."""
+        y = _c(y, np.float32)
+        M, stride = y.shape
+        assert stride >= 2 * I
+        x = np.empty((M, I), np.uint16)
+        self.lib.aio_oracle_swiglu(y.ctypes.data, M, I, stride, x.ctypes.data)
+        return x
+
+    def slice_x(self, y, off, K):
+        """x[m, k] = bf16(y[m, off + k]) for k < K."""
+        y = _c(y, np.float32)
+        M, stride = y.shape
+        assert 0 <= off and off + K <= stride
+        x = np.empty((M, K), np.uint16)
+        self.lib.aio_oracle_slice(y.ctypes.data, M, K, stride, off, x.ctypes.data)
+        return x
+
+    def prep(self, link, ys, h, h0, gammas, eps):
+        """x of one projection of a chained step from the buffers before it (``link``: a
+        synth.workloads.ChainLink); returns (x, h_out or None).  ys: fp32 y of earlier projections
+        by index; h: the two residual buffers; h0: the step's input residual stream."""
+        from synth.workloads import XOP_RMSNORM, XOP_SWIGLU, XOP_SLICE
+        if link.op == XOP_RMSNORM:
+            h_in = h0 if link.h_in < 0 else h[link.h_in]
+            r = None if link.src < 0 else ys[link.src]
+            h_out, x = self.rmsnorm(h_in, r, gammas[link.gamma], eps)
+            return x, (h_out if link.h_out >= 0 else None)
+        if link.op == XOP_SWIGLU:
+            y = ys[link.src]
+            return self.swiglu(y, y.shape[1] // 2), None
+        if link.op == XOP_SLICE:
+            return self.slice_x(ys[link.src], link.src_off, link.K), None
+        raise ValueError(link.op)
+
+    def chain_step(self, links, weights, h0, gammas, eps):
+        """A whole chained decoder step in the oracle's own arithmetic: every projection's x from
+        the oracle's earlier outputs, y rounded to fp32 as the CUDA path stores it.  weights[i] is
+        W (bf16 bits) or (q, s) for int8.  Returns (xs, ys, h) with ys in fp32."""
+        xs, ys = [], []
+        h = [None, None]
+        for link, w in zip(links, weights):
+            x, h_out = self.prep(link, ys, h, h0, gammas, eps)
+            if h_out is not None:
+                h[link.h_out] = h_out
+            y = self.linear_i8(x, *w) if isinstance(w, tuple) else self.linear_bf16(x, w)
+            xs.append(x)
+            ys.append(y.astype(np.float32))
+        return xs, ys, h
+
 
 def _default():
     return Oracle(_l())
@@ -133,3 +224,27 @@ def linear(x, W, s=None):
     if W.dtype == np.int8:
         return linear_i8(x, W, s)
     return linear_bf16(x, W)
+
+
+def double_to_bf16(v) -> int:
+    return _default().double_to_bf16(v)
+
+
+def silu(t) -> float:
+    return _default().silu(t)
+
+
+def rmsnorm(h_in, r, gamma, eps):
+    return _default().rmsnorm(h_in, r, gamma, eps)
+
+
+def swiglu(y, I):
+    return _default().swiglu(y, I)
+
+
+def slice_x(y, off, K):
+    return _default().slice_x(y, off, K)
+
+
+def chain_step(links, weights, h0, gammas, eps):
+    return _default().chain_step(links, weights, h0, gammas, eps)

@@ -26,7 +26,23 @@
  *
  * Parallelism: OpenMP over output channels n only; each output's sum order is
  * fixed, so results do not depend on the thread count.
+ *
+ * The chained decoder step (the steps on either side of the linear layers):
+ * the paper names its models (Sec. 4.2) but prints no block structure.  The
+ * reading used here is a pre-norm decoder block whose shapes match the
+ * projections: RMSNorm -> QKV -> attention -> O (+ residual) -> RMSNorm ->
+ * gate+up -> SwiGLU -> down (+ residual), and a final RMSNorm before lm_head.
+ * Attention over a context of one position (the token being decoded) gives
+ * each head's value vector, so O reads the V third of the QKV output.  Every
+ * buffer between steps has the precision the CUDA path stores: the residual
+ * stream h and every y are fp32, every projection input x is bf16 (rounded to
+ * nearest even from the exact value).  The arithmetic of each step is done in
+ * double, from those stored values:
+ *   rmsnorm:  h' = fp32(h + r);  x = bf16(h'[k] * g[k] / sqrt(mean(h'^2) + eps))
+ *   swiglu:   x = bf16(silu(y[k]) * y[I + k]),  silu(t) = t / (1 + exp(-t))
+ *   slice:    x = bf16(y[off + k])
  */
+#include <math.h>
 #include <stdint.h>
 #include <string.h>
 #include <stddef.h>
@@ -129,4 +145,82 @@ void aio_oracle_dequant_i8(const int8_t* q, const uint16_t* s, int64_t N, int64_
         double sn = aio_oracle_bf16_to_double(s[n]);
         for (int64_t k = 0; k < K; ++k) Wd[n * K + k] = sn * (double)q[n * K + k];
     }
+}
+
+/* ---------------------------------------------------------------- the chained decoder step */
+
+/* bf16 bit pattern of the double v, rounded to nearest, ties to even (no intermediate float
+ * rounding): v is rounded to a multiple of the bf16 quantum at its binade, 2^(e-8) for
+ * v = f 2^e with f in [0.5, 1), and never below 2^-133 (bf16 subnormals).  The rounded value has
+ * at most 8 significant bits, so converting it to float is exact. */
+uint16_t aio_oracle_double_to_bf16(double v) {
+    if (v != v) return 0x7FC0u;
+    if (v == 0.0) return signbit(v) ? 0x8000u : 0x0000u;
+    if (isinf(v)) return v < 0 ? 0xFF80u : 0x7F80u;
+    int e;
+    frexp(v, &e);
+    int qe = e - 8;
+    if (qe < -133) qe = -133;
+#if AIO_ORACLE_MUTANT == 7   /* rounds toward zero instead of to nearest even */
+    double r = ldexp(trunc(ldexp(v, -qe)), qe);
+#else
+    double r = ldexp(nearbyint(ldexp(v, -qe)), qe);   /* default rounding mode: nearest, ties to even */
+#endif
+    if (fabs(r) > 3.3895313892515355e38) return r < 0 ? 0xFF80u : 0x7F80u;   /* above the largest bf16 */
+    float f = (float)r;
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    return (uint16_t)(u >> 16);
+}
+
+double aio_oracle_silu(double t) {
+#if AIO_ORACLE_MUTANT == 8   /* wrong sign in the logistic */
+    return t / (1.0 + exp(t));
+#else
+    return t / (1.0 + exp(-t));
+#endif
+}
+
+/* Residual add and RMSNorm of M token rows of width K.  r may be NULL (no add); h_out may be NULL
+ * (not stored).  h_out[m, k] = fp32(h_in + r), then x[m, k] = bf16(h_out * gamma[k] * inv_rms)
+ * with inv_rms = 1 / sqrt(sum_k h_out^2 / K + eps), the sum in ascending k. */
+void aio_oracle_rmsnorm(const float* h_in, const float* r, const uint16_t* gamma, int64_t M, int64_t K, double eps,
+                        float* h_out, uint16_t* x) {
+    for (int64_t m = 0; m < M; ++m) {
+        double ss = 0.0;
+        for (int64_t k = 0; k < K; ++k) {
+            float h = r ? (float)(h_in[m * K + k] + r[m * K + k]) : h_in[m * K + k];
+            if (h_out) h_out[m * K + k] = h;
+            ss += (double)h * (double)h;
+        }
+#if AIO_ORACLE_MUTANT == 9   /* mean over K - 1 */
+        double inv = 1.0 / sqrt(ss / (double)(K - 1) + eps);
+#else
+        double inv = 1.0 / sqrt(ss / (double)K + eps);
+#endif
+        for (int64_t k = 0; k < K; ++k) {
+            float h = r ? (float)(h_in[m * K + k] + r[m * K + k]) : h_in[m * K + k];
+            x[m * K + k] = aio_oracle_double_to_bf16((double)h * aio_oracle_bf16_to_double(gamma[k]) * inv);
+        }
+    }
+}
+
+/* SwiGLU of the concatenated gate+up output: y is [M, stride] fp32 with the gate in columns
+ * [0, I) and the up projection in [I, 2I); x[m, k] = bf16(silu(gate) * up), k < I. */
+void aio_oracle_swiglu(const float* y, int64_t M, int64_t I, int64_t stride, uint16_t* x) {
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t k = 0; k < I; ++k) {
+#if AIO_ORACLE_MUTANT == 10   /* gate and up swapped */
+            double g = y[m * stride + I + k], u = y[m * stride + k];
+#else
+            double g = y[m * stride + k], u = y[m * stride + I + k];
+#endif
+            x[m * I + k] = aio_oracle_double_to_bf16(aio_oracle_silu(g) * u);
+        }
+}
+
+/* Columns [off, off + K) of y [M, stride] as bf16: x[m, k] = bf16(y[m, off + k]). */
+void aio_oracle_slice(const float* y, int64_t M, int64_t K, int64_t stride, int64_t off, uint16_t* x) {
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t k = 0; k < K; ++k) x[m * K + k] = aio_oracle_double_to_bf16((double)y[m * stride + off + k]);
 }

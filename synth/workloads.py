@@ -14,6 +14,14 @@ Recipe (all seeded, all synthetic; nothing here is the linear-layer arithmetic):
   * s   [N]     bf16 ~ U(1e-3, 1e-2)      key(seed, tag(layer), proj, KIND_S)
   where tag(layer) = family * 1000 + layer, the lm_head is layer = n_layers,
   element (m, k) of x is index m*K + k, element (n, k) of W or q is n*K + k.
+
+Chained step (the projections wired into decoder layers, see chain_links):
+  * h0  [M, H]  fp32 holding bf16 ~ N(0, 1) values (an embedding row)
+                                           key(seed, family * 1000, 0, KIND_H0)
+  * g   [H]     bf16 ~ U(0.5, 1.5), one per norm: 2l (before QKV of layer l),
+                2l + 1 (before gate+up), 2L (before lm_head)
+                                           key(seed, family * 1000 + norm, 0, KIND_GAMMA)
+  * RMSNorm epsilon RMS_EPS = 1e-5.
 """
 from __future__ import annotations
 
@@ -25,7 +33,11 @@ import numpy as np
 
 from . import codes_i8, key, normal_bf16, uniform_bf16
 
-KIND_W, KIND_X, KIND_Q, KIND_S = 0, 1, 2, 3
+KIND_W, KIND_X, KIND_Q, KIND_S, KIND_GAMMA, KIND_H0 = 0, 1, 2, 3, 4, 5
+RMS_EPS = 1e-5
+
+# How a projection of a chained step gets its x (the values of the C ABI's AIO_X_* constants).
+XOP_GIVEN, XOP_RMSNORM, XOP_SWIGLU, XOP_SLICE = 0, 1, 2, 3
 PROJ_NAMES = ("qkv", "o", "gate_up", "down", "lm_head")
 
 
@@ -151,3 +163,78 @@ def gen_rows(seed: int, wl: Workload, proj: Proj, rows: np.ndarray):
         gen_codes(seed, wl, proj, int(r), 1, out=Q[i])
         gen_scales(seed, wl, proj, int(r), 1, out=S[i:i + 1])
     return Q, S
+
+
+@dataclass(frozen=True)
+class ChainLink:
+    """Where projection i of a chained step takes its x from (structure only, no arithmetic).
+
+    op      XOP_RMSNORM: x = RMSNorm(h_in + y[src]) with norm weight `gamma`, the sum stored in
+            residual buffer h_out; XOP_SWIGLU: x = SwiGLU of y[src] (gate | up halves);
+            XOP_SLICE: x = columns [src_off, src_off + K) of y[src].
+    src     index of the projection whose y feeds x (-1: none).
+    h_in    residual buffer read (-1: the step's input h0, 0 / 1: the two residual buffers).
+    h_out   residual buffer written (-1: none).
+    """
+    op: int
+    K: int
+    src: int = -1
+    src_off: int = 0
+    h_in: int = -1
+    h_out: int = -1
+    gamma: int = -1
+
+
+def chain_links(wl: Workload) -> List[ChainLink]:
+    """Pre-norm decoder layers over the workload's projections (qkv, o, gate_up, down per layer,
+    then lm_head).  Residual adds ride on the next RMSNorm; the two residual buffers alternate so
+    that no buffer is written while another CTA may still read it (two grid barriers apart)."""
+    links: List[ChainLink] = []
+    base = {}
+    for i, p in enumerate(wl.projs):
+        base[(p.layer, p.index)] = i
+    L = max(p.layer for p in wl.projs if p.index != 4) + 1
+    for i, p in enumerate(wl.projs):
+        l = p.layer
+        if p.index == 0:      # qkv: x = RMSNorm(h), h = h_mid(l-1) + y_down(l-1)
+            if l == 0:
+                links.append(ChainLink(XOP_RMSNORM, p.K, gamma=0))
+            else:
+                links.append(ChainLink(XOP_RMSNORM, p.K, src=base[(l - 1, 3)], h_in=1, h_out=0, gamma=2 * l))
+        elif p.index == 1:    # o: attention over one position = the V third of qkv
+            q = wl.projs[base[(l, 0)]]
+            links.append(ChainLink(XOP_SLICE, p.K, src=base[(l, 0)], src_off=2 * q.N // 3))
+        elif p.index == 2:    # gate_up: x = RMSNorm(h + y_o)
+            links.append(ChainLink(XOP_RMSNORM, p.K, src=base[(l, 1)], h_in=-1 if l == 0 else 0, h_out=1,
+                                   gamma=2 * l + 1))
+        elif p.index == 3:    # down: x = SwiGLU(y_gate_up)
+            links.append(ChainLink(XOP_SWIGLU, p.K, src=base[(l, 2)]))
+        else:                 # lm_head: x = RMSNorm(h_mid(L-1) + y_down(L-1))
+            links.append(ChainLink(XOP_RMSNORM, p.K, src=base[(L - 1, 3)], h_in=1, h_out=0, gamma=2 * L))
+    return links
+
+
+def hidden(wl: Workload) -> int:
+    return wl.projs[0].K
+
+
+def gen_h0(seed: int, wl: Workload, M: int):
+    """The step's input residual stream [M, H] as fp32 (bf16-valued)."""
+    H = hidden(wl)
+    b = normal_bf16(key(seed, wl.family * 1000, 0, KIND_H0), 1.0, M * H)
+    return (b.astype(np.uint32) << 16).view(np.float32).reshape(M, H)
+
+
+def gen_gamma(seed: int, wl: Workload, norm: int, out=None):
+    return uniform_bf16(key(seed, wl.family * 1000 + norm, 0, KIND_GAMMA), 0.5, 1.5, hidden(wl), 0, out)
+
+
+def n_norms(wl: Workload) -> int:
+    return 2 * (max(p.layer for p in wl.projs if p.index != 4) + 1) + 1
+
+
+def truncated(wl: Workload, layers: int) -> Workload:
+    """The first `layers` decoder layers of wl plus its lm_head (small chained cases)."""
+    L = max(p.layer for p in wl.projs)
+    projs = [p for p in wl.projs if p.layer < layers or p.layer == L]
+    return Workload(f"{wl.name}-{layers}layer", wl.family, wl.wtype, wl.M, projs, wl.description)

@@ -2,8 +2,11 @@
 
 Each mutant is the oracle C source compiled with AIO_ORACLE_MUTANT=k:
   1 dropped term, 2 transposed operand, 3 wrong sign, 4 wrong scale index,
-  5 dequantized weight rounded to bf16 before the product, 6 lost code sign.
+  5 dequantized weight rounded to bf16 before the product, 6 lost code sign,
+  7 bf16 rounding toward zero, 8 sign error in the logistic of silu,
+  9 RMSNorm mean over K - 1, 10 SwiGLU gate and up swapped.
 """
+import math
 import struct
 from fractions import Fraction
 
@@ -58,11 +61,35 @@ def pins_hold(o: oracle.Oracle) -> bool:
     return True
 
 
+def chain_pins_hold(o: oracle.Oracle) -> bool:
+    """A few of tests/test_oracle_chain_pins.py's facts, evaluated on an arbitrary build."""
+    if o.double_to_bf16(1 + 3 * 2 ** -8) != 0x3F82 or o.double_to_bf16(1 + 2 ** -8 + 2 ** -30) != 0x3F81:
+        return False
+    if abs(o.silu(math.log(3)) - 0.75 * math.log(3)) > 1e-15:
+        return False
+    g = np.array([_bf16_int(v) for v in (1.0, 1.0, 0.5, 2.0)], np.uint16)
+    _, x = o.rmsnorm(np.array([[3.0, 4.0, 0.0, 0.0]], np.float32), None, g, 39 / 4)   # rms 4
+    if [int(v) for v in x[0]] != [0x3F40, 0x3F80, 0, 0]:
+        return False
+    t = float(np.float32(math.log(3)))
+    y = np.array([[t, 0.0, np.float32(4 / (3 * t)), 2.0]], np.float32)             # gate | up, I = 2
+    if [int(v) for v in o.swiglu(y, 2)[0]] != [0x3F80, 0]:
+        return False
+    return True
+
+
 def test_shipped_oracle_passes_pins():
-    assert pins_hold(oracle.Oracle(oracle.load()))
+    o = oracle.Oracle(oracle.load())
+    assert pins_hold(o) and chain_pins_hold(o)
 
 
 @pytest.mark.parametrize("mutant", [1, 2, 3, 4, 5, 6])
 def test_mutant_is_caught(tmp_path, mutant):
     path = ob.build(out=str(tmp_path / f"libaio_oracle_m{mutant}.so"), mutant=mutant)
     assert not pins_hold(oracle.Oracle(oracle.load(path)))
+
+
+@pytest.mark.parametrize("mutant", [7, 8, 9, 10])
+def test_chain_mutant_is_caught(tmp_path, mutant):
+    path = ob.build(out=str(tmp_path / f"libaio_oracle_m{mutant}.so"), mutant=mutant)
+    assert not chain_pins_hold(oracle.Oracle(oracle.load(path)))
