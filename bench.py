@@ -426,6 +426,8 @@ def run_ours(args, wl):
     dw.close()
     if args.pld_sweep and rank == 0:
         pld_sweep(args, peak)
+    if args.chain and rank == 0:
+        chain_lines(args, peak)
     if pg is not None:
         pg.destroy_process_group()
     return 0
@@ -469,6 +471,42 @@ def pld_sweep(args, peak):
         dw.close()
 
 
+def chain_lines(args, peak):
+    """The chained 7B-class decoder step (every x computed on the device from earlier outputs:
+    RMSNorm with residual adds, V of QKV, SwiGLU), M = 1, one persistent launch per step; one
+    JSON line per weight type after the main line."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    from synth import workloads as swl
+    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
+    for name in ("7b-bf16", "7b-int8"):
+        dw = DeviceWorkload(swl.WORKLOADS[name], seed=args.seed, max_M=1, chained=True)
+        dw.fill_chain(1)
+        wbytes = dw.weight_bytes()
+        step = dw.step_handle(1, flags)
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                aio.aio_decode_step(step, stream.cuda_stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            aio.aio_decode_step(step, stream.cuda_stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        assert aio.aio_decode_step_check(step) == 0
+        ms = e0.elapsed_time(e1) / args.steps
+        gbs = wbytes / (ms / 1e3) / 1e9
+        print(json.dumps({"sweep": "chain", "workload": f"7b-chain-{swl.WORKLOADS[name].wtype}", "M": 1,
+                          "ms_per_step": round(ms, 4), "value": round(gbs, 2), "unit": "GB/s",
+                          "frac_of_measured_peak": round(gbs / peak, 4), "tokens_per_s": round(1000.0 / ms, 2),
+                          "launches_per_step": aio.aio_decode_step_kernels(step), "steps": args.steps,
+                          "warmup": args.warmup}), flush=True)
+        dw.close()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -483,6 +521,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--pld-sweep", action="store_true",
                     help="after the main line, one line per PLD width M in {1,2,4,8} for bf16 and int8 7B steps")
+    ap.add_argument("--chain", action="store_true",
+                    help="after the main line, the chained 7B decoder step (x computed on the device), bf16 and int8")
     ap.add_argument("--step-mode", choices=["persistent", "chain"], default="persistent",
                     help="one cooperative launch per step (default) or one launch per projection")
     args = ap.parse_args()

@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 1
+#define AIO_ABI_VERSION 2
 
 typedef enum {
     AIO_OK = 0,
@@ -101,6 +101,33 @@ typedef struct {
     const void* scales;   /* [N] bf16 for int8 weights, NULL for bf16 */
     float* y;             /* [M, N] fp32 */
 } aio_proj;
+
+/*
+ * How a projection of a chained decoder step obtains its x (aio_xprep.op).  The paper names its
+ * models (Sec. 4.2) but prints no block structure; these are the steps of a pre-norm decoder block
+ * between its projections.  The device computes x at the start of the projection, after every
+ * projection before it in the step has completed, rounds it to bf16 (nearest even) and uses it;
+ * it also writes it to the projection's x buffer.  All arithmetic is fp32.
+ */
+#define AIO_X_GIVEN   0   /* x is an input the caller fills (the plain decode step) */
+#define AIO_X_RMSNORM 1   /* h = h_in + src (src may be NULL), x = h * gamma / sqrt(mean(h^2) + eps) */
+#define AIO_X_SWIGLU  2   /* x[m, k] = silu(src[m, k]) * src[m, K + k], silu(t) = t / (1 + exp(-t)) */
+#define AIO_X_SLICE   3   /* x[m, k] = src[m, src_off + k] (attention over one position: V of QKV) */
+
+typedef struct {
+    int op;               /* AIO_X_* */
+    const float* src;     /* fp32 [M, src_stride]: RMSNORM the residual to add ([M, K], stride K, or
+                             NULL), SWIGLU the gate+up output (gate in [0, K), up in [K, 2K)), SLICE
+                             the output the columns come from */
+    int src_stride;       /* elements per token row of src (SWIGLU, SLICE) */
+    int src_off;          /* SLICE: first column (multiple of 4) */
+    const float* h_in;    /* RMSNORM: residual stream [M, K] fp32 */
+    float* h_out;         /* RMSNORM: h_in + src is stored here (fp32 [M, K]) when non-NULL; it must
+                             not be h_in, and no projection of the step may read it as h_in before
+                             the next grid-wide step boundary after this projection */
+    const void* gamma;    /* RMSNORM: norm weight [K] bf16 */
+    float eps;            /* RMSNORM: >= 0 */
+} aio_xprep;
 
 /* ABI version of the loaded library (AIO_ABI_VERSION at build time). */
 int aio_abi_version(void);
@@ -209,6 +236,19 @@ aio_status aio_linear_destroy(aio_linear_t h);
  * in time.  flags: AIO_STEP_* bits.  Errors: INVALID_ARG, ALIGNMENT, STATE, UNSUPPORTED, OOM, CUDA.
  */
 aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_projs, int M, unsigned flags);
+
+/*
+ * The same, for a chained decoder step: projection i obtains its x as preps[i] says (AIO_X_*),
+ * from buffers the caller filled or earlier projections of the step wrote; preps may be NULL (all
+ * AIO_X_GIVEN).  projs[i].x receives the computed x.  A computed x is staged in shared memory, so
+ * M * (K + 32) * 2 must not exceed the staging area (35,360 bytes in the default build: M = 1 for
+ * K = 11008, M <= 4 for K = 4096): UNSUPPORTED otherwise.  src, h_in, h_out and gamma must be
+ * 16-byte aligned, src_stride and src_off multiples of 4: ALIGNMENT otherwise.  A missing pointer,
+ * a column range outside src_stride, h_out == h_in or a negative eps: INVALID_ARG.  Device errors
+ * are reported as for aio_decode_step_create.
+ */
+aio_status aio_decode_step_create_chained(aio_step_t* out, const aio_proj* projs, const aio_xprep* preps,
+                                          int n_projs, int M, unsigned flags);
 
 /* Enqueue one decode step on stream (one graph launch with AIO_STEP_GRAPH). */
 aio_status aio_decode_step(aio_step_t step, void* stream);

@@ -42,6 +42,11 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
+AIO_ABI_VERSION = 2
+AIO_X_GIVEN = 0
+AIO_X_RMSNORM = 1
+AIO_X_SWIGLU = 2
+AIO_X_SLICE = 3
 for _name, _val in re.findall(r"#define\s+(AIO_\w+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", _hdr):
     if _name in globals() and globals()[_name] != int(_val, 0):
         raise ImportError(f"binding constant {_name} disagrees with include/aio.h")
@@ -58,6 +63,12 @@ class AioError(RuntimeError):
 class aio_proj(ctypes.Structure):
     _fields_ = [("h", ctypes.c_void_p), ("x", ctypes.c_void_p), ("W", ctypes.c_void_p),
                 ("scales", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
+class aio_xprep(ctypes.Structure):
+    _fields_ = [("op", ctypes.c_int), ("src", ctypes.c_void_p), ("src_stride", ctypes.c_int),
+                ("src_off", ctypes.c_int), ("h_in", ctypes.c_void_p), ("h_out", ctypes.c_void_p),
+                ("gamma", ctypes.c_void_p), ("eps", ctypes.c_float)]
 
 
 _vp, _int, _u = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint
@@ -78,6 +89,8 @@ _SIGS = {
     "aio_linear_reset": (_int, [_vp]),
     "aio_linear_destroy": (_int, [_vp]),
     "aio_decode_step_create": (_int, [ctypes.POINTER(_vp), ctypes.POINTER(aio_proj), _int, _int, _u]),
+    "aio_decode_step_create_chained": (_int, [ctypes.POINTER(_vp), ctypes.POINTER(aio_proj),
+                                              ctypes.POINTER(aio_xprep), _int, _int, _u]),
     "aio_decode_step": (_int, [_vp, _vp]),
     "aio_decode_step_kernels": (_int, [_vp, ctypes.POINTER(_int)]),
     "aio_decode_step_check": (_int, [_vp, ctypes.POINTER(_int)]),
@@ -168,6 +181,18 @@ def aio_decode_step_create(projs, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP
     arr = (aio_proj * len(projs))(*[aio_proj(*p) for p in projs])
     s = _vp()
     _check(_lib.aio_decode_step_create(ctypes.byref(s), arr, len(projs), M, flags), "aio_decode_step_create")
+    return s.value
+
+
+def aio_decode_step_create_chained(projs, preps, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP_PERSISTENT) -> int:
+    """projs as for aio_decode_step_create; preps: one (op, src, src_stride, src_off, h_in, h_out,
+    gamma, eps) tuple per projection, addresses as integers or None."""
+    assert len(preps) == len(projs)
+    arr = (aio_proj * len(projs))(*[aio_proj(*p) for p in projs])
+    parr = (aio_xprep * len(preps))(*[aio_xprep(*x) for x in preps])
+    s = _vp()
+    _check(_lib.aio_decode_step_create_chained(ctypes.byref(s), arr, parr, len(projs), M, flags),
+           "aio_decode_step_create_chained")
     return s.value
 
 

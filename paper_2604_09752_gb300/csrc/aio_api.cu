@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdarg>
 #include <cstdint>
 #include <cstdio>
@@ -385,7 +386,47 @@ static aio_status step_launch_all(aio_step* s, cudaStream_t stream) {
     return AIO_OK;
 }
 
-aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_projs, int M, unsigned flags) {
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Host checks of one projection's x preparation (see aio_decode_step_create_chained).
+static aio_status validate_prep(const aio_linear* h, const aio_xprep& x, int M) {
+    if (x.op == AIO_X_GIVEN) return AIO_OK;
+    if (x.op != AIO_X_RMSNORM && x.op != AIO_X_SWIGLU && x.op != AIO_X_SLICE)
+        return fail(AIO_ERR_INVALID_ARG, "unknown x preparation %d", x.op);
+    const int K = h->K;
+    if (static_cast<long long>(M) * (K + aio::kXsPad) * 2 > aio::kXsBytes)
+        return fail(AIO_ERR_UNSUPPORTED, "a computed x needs M (K + 32) 2 <= %d bytes (M=%d, K=%d)", aio::kXsBytes, M, K);
+    if (x.op == AIO_X_RMSNORM) {
+        if (!x.h_in || !x.gamma) return fail(AIO_ERR_INVALID_ARG, "RMSNORM needs h_in and gamma");
+        if (!(x.eps >= 0.0f) || !std::isfinite(x.eps)) return fail(AIO_ERR_INVALID_ARG, "eps must be finite and >= 0");
+        if (x.h_out && (x.h_out == x.h_in || x.h_out == x.src))
+            return fail(AIO_ERR_INVALID_ARG, "h_out must differ from h_in and src");
+        if (!aligned16(x.h_in) || !aligned16(x.gamma) || !aligned16(x.h_out) || !aligned16(x.src))
+            return fail(AIO_ERR_ALIGNMENT, "h_in, h_out, src and gamma must be 16-byte aligned");
+        return AIO_OK;
+    }
+    if (!x.src) return fail(AIO_ERR_INVALID_ARG, "SWIGLU and SLICE need src");
+    if (!aligned16(x.src) || x.src_stride % 4 != 0 || x.src_off % 4 != 0)
+        return fail(AIO_ERR_ALIGNMENT, "src must be 16-byte aligned, src_stride and src_off multiples of 4");
+    const long long need = x.op == AIO_X_SWIGLU ? 2LL * K : static_cast<long long>(x.src_off) + K;
+    if (x.src_off < 0 || x.src_stride < need)
+        return fail(AIO_ERR_INVALID_ARG, "columns [%lld, %lld) outside src_stride %d", need - K, need, x.src_stride);
+    return AIO_OK;
+}
+
+static void apply_prep(aio::ProjDesc& d, const aio_xprep& x) {
+    d.xop = x.op;
+    d.xsrc = x.src;
+    d.xsrc_stride = x.op == AIO_X_RMSNORM ? d.K : x.src_stride;
+    d.xsrc_off = x.src_off;
+    d.h_in = x.h_in;
+    d.h_out = x.h_out;
+    d.gamma = static_cast<const uint16_t*>(x.gamma);
+    d.eps = x.eps;
+}
+
+static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_xprep* preps, int n_projs, int M,
+                              unsigned flags) {
     if (!out) return fail(AIO_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
     if (!projs || n_projs < 1) return fail(AIO_ERR_INVALID_ARG, "need at least one projection");
@@ -409,6 +450,8 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
         if (persistent && p.h->wt != wt0)
             return fail(AIO_ERR_UNSUPPORTED, "a persistent step needs one weight type (projection %d differs)", i);
         if ((st = validate_run(p.h, p.x, M, p.W, p.scales, p.y)) != AIO_OK)
+            return fail(st, "projection %d: %s", i, g_last_error);
+        if (preps && (st = validate_prep(p.h, preps[i], M)) != AIO_OK)
             return fail(st, "projection %d: %s", i, g_last_error);
         offs[i] = total;
         total += aio::workspace_bytes(p.h->geo, M);
@@ -451,6 +494,7 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     for (int i = 0; i < n_projs; ++i) {
         const aio_proj& p = projs[i];
         descs.push_back(make_desc(p.h, p.x, p.W, p.scales, p.y, reinterpret_cast<float*>(base + offs[i])));
+        if (preps) apply_prep(descs.back(), preps[i]);
         s->chain.push_back(single_args(p.h, descs.back(), M, s->errs + i));
         s->chain_i8.push_back(p.h->wt == AIO_W_INT8_PERCHANNEL ? 1 : 0);
     }
@@ -501,6 +545,15 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
     }
     *out = s;
     return AIO_OK;
+}
+
+aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_projs, int M, unsigned flags) {
+    return step_create(out, projs, nullptr, n_projs, M, flags);
+}
+
+aio_status aio_decode_step_create_chained(aio_step_t* out, const aio_proj* projs, const aio_xprep* preps,
+                                          int n_projs, int M, unsigned flags) {
+    return step_create(out, projs, preps, n_projs, M, flags);
 }
 
 static aio_status valid_step(aio_step_t s) {

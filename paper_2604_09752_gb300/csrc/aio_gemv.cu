@@ -347,6 +347,7 @@ struct Proj {
     int Tq, Tr;
     int M, K, N, NKT;
     int rowmajor, uniform;
+    int xop;
 };
 
 __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
@@ -364,6 +365,7 @@ __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
     p.NKT = d->NKT;
     p.rowmajor = d->rowmajor;
     p.uniform = d->uniform;
+    p.xop = d->xop;
     return p;
 }
 
@@ -792,6 +794,132 @@ __device__ __forceinline__ unsigned cta_arrive(unsigned* cta_count, unsigned* gl
     return __shfl_sync(0xffffffffu, g, 0);
 }
 
+// ------------------------------------------------------------------ x of a chained step
+__device__ __forceinline__ void named_barrier_sync() {
+    asm volatile("bar.sync 1, %0;" ::"n"(kThreads) : "memory");
+}
+
+// Data another CTA wrote before the grid barrier: read at L2, never from a stale L1 line.
+__device__ __forceinline__ float4 ldcg4(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
+
+__device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi) {
+    return static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(lo))) |
+           (static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(hi))) << 16);
+}
+
+// Four consecutive x values of one token at k = 4i, rounded to bf16: into this CTA's staged copy,
+// and from CTA 0 into the projection's x buffer as well.
+__device__ __forceinline__ void put_x4(uint16_t* xs_row, uint16_t* xg_row, int i, float a, float b, float c, float d,
+                                       bool cta0) {
+    const uint2 v = make_uint2(bf16x2_rn(a, b), bf16x2_rn(c, d));
+    *reinterpret_cast<uint2*>(xs_row + 4 * i) = v;
+    if (cta0) *reinterpret_cast<uint2*>(xg_row + 4 * i) = v;
+}
+
+// silu(t) = t / (1 + e^-t), evaluated with e^-|t| so that the exponential never overflows (for
+// t < 0 it is t e^t / (1 + e^t)).
+__device__ __forceinline__ float silu(float t) {
+    const float e = expf(-fabsf(t));
+    return t >= 0.0f ? t / (1.0f + e) : t * e / (1.0f + e);
+}
+
+// x of a projection in a chained decoder step, computed by every thread of the CTA into the staged
+// copy xs (row stride xs_stride) after the grid barrier, from buffers earlier projections wrote:
+//   RMSNorm: h = h_in + xsrc (fp32 add; CTA 0 stores h in h_out), x = bf16(h * gamma / rms(h)),
+//            rms(h) = sqrt(sum h^2 / K + eps), the sum reduced in a fixed order;
+//   SwiGLU:  x = bf16(silu(g) * u), g = xsrc[m, k], u = xsrc[m, K + k];
+//   slice:   x = bf16(xsrc[m, off + k]).
+// red holds kWarps x kMaxM floats of shared scratch.  Ends with a CTA-wide barrier.
+template <int MT>
+__device__ __forceinline__ void prep_x(const ProjDesc* d, uint16_t* xs, int xs_stride, float* red, int warp,
+                                       int lane) {
+    const int tid = warp * 32 + lane;
+    const int K = d->K, n4 = K / 4, op = d->xop;
+    const bool cta0 = blockIdx.x == 0;
+    uint16_t* xg = const_cast<uint16_t*>(d->x);
+    const float* src = d->xsrc;
+    if (op == kXRmsNorm) {
+        const float* hin = d->h_in;
+        float* hout = d->h_out;
+        float ss[MT];
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            float acc = 0.0f;
+#pragma unroll 4
+            for (int i = tid; i < n4; i += kThreads) {
+                float4 a = ldcg4(hin + m * K + 4 * i);
+                if (src) {
+                    const float4 b = ldcg4(src + m * K + 4 * i);
+                    a.x += b.x;
+                    a.y += b.y;
+                    a.z += b.z;
+                    a.w += b.w;
+                }
+                acc = fmaf(a.x, a.x, acc);
+                acc = fmaf(a.y, a.y, acc);
+                acc = fmaf(a.z, a.z, acc);
+                acc = fmaf(a.w, a.w, acc);
+                if (cta0 && hout) *reinterpret_cast<float4*>(hout + m * K + 4 * i) = a;
+            }
+            ss[m] = acc;
+        }
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            float v = ss[m];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            if (lane == 0) red[warp * kMaxM + m] = v;
+        }
+        named_barrier_sync();
+        const uint2* g4 = reinterpret_cast<const uint2*>(d->gamma);
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            float tot = 0.0f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) tot += red[w * kMaxM + m];
+            const float inv = 1.0f / sqrtf(tot / static_cast<float>(K) + d->eps);
+#pragma unroll 4
+            for (int i = tid; i < n4; i += kThreads) {
+                float4 a = ldcg4(hin + m * K + 4 * i);
+                if (src) {
+                    const float4 b = ldcg4(src + m * K + 4 * i);
+                    a.x += b.x;
+                    a.y += b.y;
+                    a.z += b.z;
+                    a.w += b.w;
+                }
+                const uint2 gb = __ldg(g4 + i);
+                put_x4(xs + m * xs_stride, xg + m * K, i, a.x * __uint_as_float(gb.x << 16) * inv,
+                       a.y * __uint_as_float(gb.x & 0xFFFF0000u) * inv, a.z * __uint_as_float(gb.y << 16) * inv,
+                       a.w * __uint_as_float(gb.y & 0xFFFF0000u) * inv, cta0);
+            }
+        }
+    } else if (op == kXSwiGlu) {
+        const int stride = d->xsrc_stride;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+#pragma unroll 4
+            for (int i = tid; i < n4; i += kThreads) {
+                const float4 g = ldcg4(src + m * stride + 4 * i);
+                const float4 u = ldcg4(src + m * stride + K + 4 * i);
+                put_x4(xs + m * xs_stride, xg + m * K, i, silu(g.x) * u.x, silu(g.y) * u.y, silu(g.z) * u.z,
+                       silu(g.w) * u.w, cta0);
+            }
+        }
+    } else {
+        const int stride = d->xsrc_stride, off = d->xsrc_off;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+#pragma unroll 4
+            for (int i = tid; i < n4; i += kThreads) {
+                const float4 v = ldcg4(src + m * stride + off + 4 * i);
+                put_x4(xs + m * xs_stride, xg + m * K, i, v.x, v.y, v.z, v.w, cta0);
+            }
+        }
+    }
+    named_barrier_sync();
+}
+
 // The stream kernel: one CTA per SM, every warp streams its segment of every projection through
 // its own bulk-copy ring.  All per-tile bookkeeping is incremental 32-bit arithmetic; divisions
 // happen once per chunk (issue) or once per projection (consume).
@@ -812,6 +940,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     // x of the current projection, staged once per CTA when it fits (one bulk copy by warp 0).
     uint64_t* xbar = reinterpret_cast<uint64_t*>(smem + kSyncOffset + 16);
     uint16_t* xs = reinterpret_cast<uint16_t*>(smem + kXsOffset);
+    float* red = reinterpret_cast<float*>(smem + kAuxOffset);   // x preparation scratch
 
     griddep_launch_dependents();
 
@@ -828,7 +957,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         mbar_init(xbar, 1);
         fence_mbar_init();
     }
-    __syncthreads();   // the only CTA-wide barrier: barriers and sync words are initialised
+    __syncthreads();   // barriers and sync words are initialised (later CTA-wide barriers: prep_x only)
     const uint64_t pol = policy_evict_first();
     const I8Consts kc = i8_consts();
 
@@ -889,7 +1018,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         // CTA has then finished reading the previous x and fenced its reads against async writes):
         // one bulk copy per token row.
         auto stage_x = [&]() {
-            if (stage && lane == 0) {
+            if (stage && P.xop == kXGiven && lane == 0) {
                 mbar_expect_tx(xbar, static_cast<uint32_t>(P.M * P.K * 2));
                 for (int m = 0; m < P.M; ++m)
                     bulk_g2s_plain(xs + m * xs_stride, P.x + static_cast<size_t>(m) * P.K,
@@ -915,13 +1044,22 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 dead = true;
             }
         }
-        if (stage) {
+        if (stage && P.xop == kXGiven) {
             // every warp waits for the staged x (also so that no copy is in flight at exit)
             if (!__all_sync(0xffffffffu, mbar_wait(xbar, xphase, s.wait_limit_ns)) && !dead) {
                 if (lane == 0) atomicExch(s.err, kDevErrTimeout);
                 dead = true;
             }
             xphase ^= 1u;
+        }
+        if (P.xop != kXGiven) {
+            // chained step: every warp of the CTA computes x (uniform over the CTA, dead or not)
+            if (stage) {
+                prep_x<MT>(proj_desc(s, p), xs, xs_stride, red, warp, lane);
+            } else if (!dead) {
+                if (lane == 0) atomicCAS(s.err, 0, kDevErrPrep);
+                dead = true;
+            }
         }
         ahead = 0;
         if (!dead) {

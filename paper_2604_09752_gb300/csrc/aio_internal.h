@@ -51,16 +51,22 @@ constexpr int kMaxStages = kStages > kStagesI8 ? kStages : kStagesI8;
 static_assert(kSlotBytes % 8192 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
 static_assert(kSlotBytesI8 % 4096 == 0 && kStagesI8 >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
 constexpr int kSyncOffset = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;  // CTA-level sync words
-constexpr int kXsOffset = kSyncOffset + 32;        // sync words (16 B), the x barrier (8 B), padding
+constexpr int kMaxM = 8;
+constexpr int kAuxOffset = kSyncOffset + 32;       // sync words (16 B), the x barrier (8 B), padding
+constexpr int kAuxBytes = kWarps * kMaxM * 4;      // per-warp, per-token partial sums (x preparation)
+constexpr int kXsOffset = kAuxOffset + (kAuxBytes + 15) / 16 * 16;
 constexpr int kXsPad = 32;                         // elements between staged x rows beyond K (64 B)
 constexpr int kXsBytes = 227 * 1024 - kXsOffset;   // x staged in shared memory when M * (K + kXsPad) * 2 fits
 constexpr int kSmemBytes = kXsOffset + kXsBytes;
-constexpr int kMaxM = 8;
 static_assert(kSmemBytes <= 227 * 1024, "ring does not fit in shared memory");
 static_assert(kXsOffset % 16 == 0, "bulk-copy destination alignment");
 
 constexpr int kDevErrTimeout = 1;       // a bulk-copy wait expired
 constexpr int kDevErrGridTimeout = 2;   // a wait for the previous projection expired
+constexpr int kDevErrPrep = 3;          // x preparation asked for a projection whose x is not staged
+
+// How a projection's x is obtained (the values of AIO_X_*).
+constexpr int kXGiven = 0, kXRmsNorm = 1, kXSwiGlu = 2, kXSlice = 3;
 
 // One projection of a launch; read-only while the kernel runs.  Geometry:
 //   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles;
@@ -76,6 +82,16 @@ struct ProjDesc {
     int K, N, NG, NKT;
     int rowmajor;             // 1: W is row-major [N, K]
     int uniform;              // 1: packed, N % 8 == 0 and K % 256 == 0, so tile t is bytes [t, t+1) * tile size
+    // x preparation in a chained step (xop != kXGiven): x is computed by every CTA into its staged
+    // copy (and by CTA 0 into x itself) from buffers earlier projections wrote.
+    const float* xsrc;        // RMSNorm: added to h_in (may be null); SwiGLU, slice: the y read
+    const float* h_in;        // RMSNorm: residual stream [M, K]
+    float* h_out;             // RMSNorm: h_in + xsrc, written by CTA 0 (may be null)
+    const uint16_t* gamma;    // RMSNorm: [K] bf16
+    int xop;
+    int xsrc_stride;          // elements per token row of xsrc
+    int xsrc_off;             // slice: first column
+    float eps;                // RMSNorm
 };
 static_assert(sizeof(ProjDesc) % 16 == 0, "descriptor array stride");
 

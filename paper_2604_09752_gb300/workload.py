@@ -8,6 +8,11 @@ tiles each weight matrix on the device.
 Buffers: one bf16 x arena and one fp32 y arena hold every projection's x [M, K]
 and y [M, N] back to back (each slice 256-byte aligned), so a whole step's
 inputs and outputs move with one host<->device copy each.
+
+A chained workload (``chained=True``) wires the projections into decoder layers
+(synth.workloads.chain_links): the device computes every projection's x from
+earlier outputs, so the step's only inputs are the residual stream h0 and the
+norm weights.
 """
 from __future__ import annotations
 
@@ -45,7 +50,8 @@ class DeviceWorkload:
     """
 
     def __init__(self, wl: swl.Workload, seed: int = 0, max_M: int = 8, layout: str = "packed",
-                 device: Optional[torch.device] = None, projs: Optional[List[swl.Proj]] = None):
+                 device: Optional[torch.device] = None, projs: Optional[List[swl.Proj]] = None,
+                 chained: bool = False):
         assert layout in ("packed", "rowmajor")
         self.wl = wl
         self.seed = seed
@@ -72,6 +78,15 @@ class DeviceWorkload:
         self.y_arena = torch.zeros(y_bytes, dtype=torch.uint8, device=self.device)
         self.bufs: List[_ProjBuf] = []
         self._load_weights(offs)
+        self.chained = chained
+        if chained:
+            self.links = swl.chain_links(swl.Workload(wl.name, wl.family, wl.wtype, wl.M, self.projs))
+            H = self.projs[0].K
+            hb = _round(max_M * H * 4)
+            # h0, the two residual buffers, then the norm weights [n_norms, H] bf16
+            self.n_norms = max(l.gamma for l in self.links) + 1
+            self.h_arena = torch.zeros(3 * hb + _round(self.n_norms * H * 2), dtype=torch.uint8, device=self.device)
+            self._hb = hb
 
     # ------------------------------------------------------------------ loading
     def _load_weights(self, offs):
@@ -115,6 +130,49 @@ class DeviceWorkload:
         torch.cuda.synchronize(self.device)
         return host
 
+    def fill_chain(self, M: Optional[int] = None):
+        """Write the chained step's inputs: h0 [M, H] (fp32) and every norm weight [H] (bf16)."""
+        assert self.chained
+        M = M or self.wl.M
+        H = self.projs[0].K
+        host = torch.zeros(self.h_arena.numel(), dtype=torch.uint8, pin_memory=True)
+        h0 = swl.gen_h0(self.seed, self.wl, M)
+        host[: M * H * 4].copy_(torch.from_numpy(h0.view("uint8").reshape(-1)))
+        g = host[3 * self._hb:].view(torch.int16)
+        for j in range(self.n_norms):
+            swl.gen_gamma(self.seed, self.wl, j, out=g.data_ptr() + j * H * 2)
+        self.h_arena.copy_(host)
+        torch.cuda.synchronize(self.device)
+        return h0
+
+    def h_ptr(self, j: int) -> int:
+        """-1: the input h0; 0 / 1: the residual buffers."""
+        return self.h_arena.data_ptr() + (j + 1) * self._hb
+
+    def h(self, j: int, M: int) -> torch.Tensor:
+        H = self.projs[0].K
+        o = (j + 1) * self._hb
+        return self.h_arena[o: o + M * H * 4].view(torch.float32).view(M, H)
+
+    def gamma_ptr(self, j: int) -> int:
+        return self.h_arena.data_ptr() + 3 * self._hb + j * self.projs[0].K * 2
+
+    def gamma(self, j: int) -> torch.Tensor:
+        H = self.projs[0].K
+        o = 3 * self._hb + j * H * 2
+        return self.h_arena[o: o + H * 2].view(torch.int16)
+
+    def _preps(self):
+        out = []
+        for i, (b, l) in enumerate(zip(self.bufs, self.links)):
+            src = self.y_ptr(l.src) if l.src >= 0 else None
+            if l.op == swl.XOP_RMSNORM:
+                out.append((l.op, src, b.proj.K, 0, self.h_ptr(l.h_in), self.h_ptr(l.h_out) if l.h_out >= 0 else None,
+                            self.gamma_ptr(l.gamma), swl.RMS_EPS))
+            else:
+                out.append((l.op, src, self.bufs[l.src].proj.N, l.src_off, None, None, None, 0.0))
+        return out
+
     # ------------------------------------------------------------------ views and calls
     def x_ptr(self, i: int) -> int:
         return self.x_arena.data_ptr() + self.bufs[i].x_off
@@ -137,12 +195,17 @@ class DeviceWorkload:
                            b.scales.data_ptr() if b.scales is not None else None, self.y_ptr(i), s)
 
     def step_handle(self, M: int, flags: int = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT) -> int:
+        """The step over every projection: chained (x computed on the device) for a chained
+        workload, else with every x an input."""
         key = (M, flags)
         if key not in self._steps:
             projs = [(b.handle, self.x_ptr(i), b.W.data_ptr(),
                       b.scales.data_ptr() if b.scales is not None else None, self.y_ptr(i))
                      for i, b in enumerate(self.bufs)]
-            self._steps[key] = aio.aio_decode_step_create(projs, M, flags)
+            if self.chained:
+                self._steps[key] = aio.aio_decode_step_create_chained(projs, self._preps(), M, flags)
+            else:
+                self._steps[key] = aio.aio_decode_step_create(projs, M, flags)
         return self._steps[key]
 
     def step(self, M: int, flags: int = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT, stream: Optional[int] = None):
