@@ -57,8 +57,10 @@ def measured_peak():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for f in ("aio_gemv.cu", "aio_internal.h"):
-        h.update(open(os.path.join(ROOT, "paper_2604_09752_gb300", "csrc", f), "rb").read())
+    for f in ("aio_stream.cuh", "aio_gemv.cu", "aio_chain.cu", "aio_internal.h"):
+        path = os.path.join(ROOT, "paper_2604_09752_gb300", "csrc", f)
+        if os.path.exists(path):
+            h.update(open(path, "rb").read())
     return h.hexdigest()[:16]
 
 

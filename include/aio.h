@@ -240,9 +240,9 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
 /*
  * The same, for a chained decoder step: projection i obtains its x as preps[i] says (AIO_X_*),
  * from buffers the caller filled or earlier projections of the step wrote; preps may be NULL (all
- * AIO_X_GIVEN).  projs[i].x receives the computed x.  A computed x is staged in shared memory, so
- * M * (K + 32) * 2 must not exceed the staging area (35,360 bytes in the default build: M = 1 for
- * K = 11008, M <= 4 for K = 4096): UNSUPPORTED otherwise.  src, h_in, h_out and gamma must be
+ * AIO_X_GIVEN).  projs[i].x receives the computed x.  A chained step takes M <= 4, and a computed x
+ * is staged in shared memory, so M * (K + 32) * 2 must not exceed the staging area (35,360 bytes in
+ * the default build: M = 1 for K = 11008, M <= 4 for K = 4096): UNSUPPORTED otherwise.  src, h_in, h_out and gamma must be
  * 16-byte aligned, src_stride and src_off multiples of 4: ALIGNMENT otherwise.  A missing pointer,
  * a column range outside src_stride, h_out == h_in or a negative eps: INVALID_ARG.  Device errors
  * are reported as for aio_decode_step_create.

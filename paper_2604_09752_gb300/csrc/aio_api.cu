@@ -117,6 +117,7 @@ struct aio_step {
     int device, M, n;
     unsigned flags;
     bool persistent;
+    bool chained;                        // some projection computes its x (the chained kernels run)
     bool i8;                             // weight type of every projection (persistent mode)
     int grid;
     std::vector<aio::StreamArgs> chain;  // per-projection launches (chain mode)
@@ -376,12 +377,12 @@ static void step_free(aio_step* s) {
 
 static aio_status step_launch_all(aio_step* s, cudaStream_t stream) {
     if (s->persistent) {
-        AIO_CUDA(aio::launch_stream(s->whole, s->i8, s->grid, stream, false, true));
+        AIO_CUDA(aio::launch_stream(s->whole, s->i8, s->grid, stream, false, true, s->chained));
         return AIO_OK;
     }
     for (int i = 0; i < s->n; ++i) {
         const bool pdl = i > 0 && (s->flags & AIO_STEP_PDL);
-        AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false));
+        AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false, s->chained));
     }
     return AIO_OK;
 }
@@ -459,9 +460,13 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
     aio_status st = check_device(dev);
     if (st != AIO_OK) return st;
     const int grid = projs[0].h->geo.grid;
+    bool chained = false;
+    for (int i = 0; preps && i < n_projs; ++i) chained = chained || preps[i].op != AIO_X_GIVEN;
+    if (chained && M > aio::kMaxChainM)
+        return fail(AIO_ERR_UNSUPPORTED, "a chained step supports M <= %d (M=%d)", aio::kMaxChainM, M);
     if (persistent) {
         int blocks = 0;
-        AIO_CUDA(aio::occupancy(wt0 == AIO_W_INT8_PERCHANNEL, M, &blocks));
+        AIO_CUDA(aio::occupancy(wt0 == AIO_W_INT8_PERCHANNEL, M, chained, &blocks));
         if (blocks < 1) return fail(AIO_ERR_UNSUPPORTED, "the stream kernel cannot be resident on an SM");
     }
     const size_t desc_off = total;
@@ -479,6 +484,7 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
     s->n = n_projs;
     s->flags = flags;
     s->persistent = persistent;
+    s->chained = chained;
     s->i8 = wt0 == AIO_W_INT8_PERCHANNEL;
     s->grid = grid;
     s->ws_bytes = total;

@@ -124,8 +124,12 @@ size_t workspace_bytes(const Geometry& g, int M);
 
 cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared memory)
 // pdl: programmatic dependent launch; coop: cooperative launch (all CTAs co-resident).
-cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop);
-cudaError_t occupancy(bool i8, int M, int* blocks_per_sm);
+using StreamFn = void (*)(const StreamArgs);
+constexpr int kMaxChainM = 4;   // token rows of a chained step (its kernels are instantiated for M <= 4)
+StreamFn chain_stream_fn(bool i8, int M);   // aio_chain.cu
+cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop,
+                          bool chained = false);
+cudaError_t occupancy(bool i8, int M, bool chained, int* blocks_per_sm);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
 cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s);
 

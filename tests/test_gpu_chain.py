@@ -163,10 +163,12 @@ def test_full_7b_chain_sampled(aio):
 def test_chained_step_rejects_bad_preparations(aio):
     h = aio.aio_linear_create(11008, 64, aio.AIO_W_BF16, 2, 0)
     h2 = aio.aio_linear_create(256, 64, aio.AIO_W_BF16, 2, 0)
+    h8 = aio.aio_linear_create(256, 64, aio.AIO_W_BF16, 8, 0)
     buf = torch.zeros(1 << 22, dtype=torch.uint8, device="cuda")
     p = buf.data_ptr()
     proj = [(h, p, p + (1 << 21), None, p + 65536)]
     proj2 = [(h2, p, p + (1 << 21), None, p + 65536)]
+    proj8 = [(h8, p, p + (1 << 21), None, p + 65536)]
     cases = [
         (proj, [(aio.AIO_X_SWIGLU, p + 4096, 2 * 11008, 0, None, None, None, 0.0)], 2, aio.AIO_ERR_UNSUPPORTED),
         (proj2, [(9, p + 4096, 512, 0, None, None, None, 0.0)], 1, aio.AIO_ERR_INVALID_ARG),
@@ -178,6 +180,7 @@ def test_chained_step_rejects_bad_preparations(aio):
         (proj2, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8192, p + 8192, p, 1e-5)], 1, aio.AIO_ERR_INVALID_ARG),
         (proj2, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8192, None, p, -1.0)], 1, aio.AIO_ERR_INVALID_ARG),
         (proj2, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8200, None, p, 1e-5)], 1, aio.AIO_ERR_ALIGNMENT),
+        (proj8, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8192, None, p, 1e-5)], 5, aio.AIO_ERR_UNSUPPORTED),
     ]
     for pr, prep, M, status in cases:
         with pytest.raises(aio.AioError) as e:
@@ -185,3 +188,4 @@ def test_chained_step_rejects_bad_preparations(aio):
         assert e.value.status == status, (prep, e.value)
     aio.aio_linear_destroy(h)
     aio.aio_linear_destroy(h2)
+    aio.aio_linear_destroy(h8)
