@@ -17,6 +17,8 @@ Functions and the passages they follow:
   * pack_tiles / unpack_tiles  the tiled weight layout the CUDA packer must
                              produce (a pure permutation; see layout.py).
   * double_to_bf16(v)        round a double to bf16, nearest-even.
+  * attention(q, k, v, L)    decode attention of M new tokens over a KV cache of
+                             L positions (the long-context path, Sec. 3.3, Sec. 5.1).
   * silu(t), rmsnorm(...), swiglu(...), slice_x(...)
                              the steps between the projections of a chained
                              decoder step; chain_step(...) runs a whole chained
@@ -70,6 +72,8 @@ def load(path: str = LIB_PATH):
     lib.aio_oracle_swiglu.argtypes = [vp, i64, i64, i64, vp]
     lib.aio_oracle_slice.restype = None
     lib.aio_oracle_slice.argtypes = [vp, i64, i64, i64, i64, vp]
+    lib.aio_oracle_attention.restype = None
+    lib.aio_oracle_attention.argtypes = [vp, i64, vp, vp, i64, i64, i64, i64, i64, vp]
     return lib
 
 
@@ -168,6 +172,21 @@ class Oracle:
         self.lib.aio_oracle_slice(y.ctypes.data, M, K, stride, off, x.ctypes.data)
         return x
 
+    def attention(self, q, k, v, L, M=None):
+        """Decode attention: q [M, n_heads d] fp32 (rows may be wider: only the first n_heads d
+        columns are read), k, v [n_heads, L_max, d] bf16 bits; the M new tokens sit at positions
+        L - M .. L - 1 and attend causally.  Returns out [M, n_heads d] in double."""
+        q = _c(q, np.float32)
+        k = _c(k, np.uint16)
+        v = _c(v, np.uint16)
+        n_heads, L_max, d = k.shape
+        M = q.shape[0] if M is None else M
+        assert v.shape == k.shape and 1 <= L <= L_max and M <= L and q.shape[1] >= n_heads * d
+        out = np.empty((M, n_heads * d), np.float64)
+        self.lib.aio_oracle_attention(q.ctypes.data, q.shape[1], k.ctypes.data, v.ctypes.data, n_heads, d, L_max, L, M,
+                                      out.ctypes.data)
+        return out
+
     def prep(self, link, ys, h, h0, gammas, eps):
         """x of one projection of a chained step from the buffers before it (``link``: a
         synth.workloads.ChainLink); returns (x, h_out or None).  ys: fp32 y of earlier projections
@@ -248,3 +267,7 @@ def slice_x(y, off, K):
 
 def chain_step(links, weights, h0, gammas, eps):
     return _default().chain_step(links, weights, h0, gammas, eps)
+
+
+def attention(q, k, v, L, M=None):
+    return _default().attention(q, k, v, L, M)

@@ -41,6 +41,13 @@
  *   rmsnorm:  h' = fp32(h + r);  x = bf16(h'[k] * g[k] / sqrt(mean(h'^2) + eps))
  *   swiglu:   x = bf16(silu(y[k]) * y[I + k]),  silu(t) = t / (1 + exp(-t))
  *   slice:    x = bf16(y[off + k])
+ *
+ * Decode attention over a KV cache (the long-context half of the paper's routing, Sec. 3.3,
+ * Sec. 5.1: standard contexts up to 2K tokens, long ones up to 32K).  For each head h and new
+ * token m of M (positions L - M + m of a cache holding L positions), with d-dimensional heads:
+ *   s_j = q[m, h] . k[h, j] / sqrt(d)  for j <= L - M + m   (causal among the new tokens)
+ *   out[m, h] = sum_j softmax(s)_j v[h, j]
+ * in double, from fp32 q and bf16 cache entries.
  */
 #include <math.h>
 #include <stdint.h>
@@ -223,4 +230,52 @@ void aio_oracle_swiglu(const float* y, int64_t M, int64_t I, int64_t stride, uin
 void aio_oracle_slice(const float* y, int64_t M, int64_t K, int64_t stride, int64_t off, uint16_t* x) {
     for (int64_t m = 0; m < M; ++m)
         for (int64_t k = 0; k < K; ++k) x[m * K + k] = aio_oracle_double_to_bf16((double)y[m * stride + off + k]);
+}
+
+/* ---------------------------------------------------------------- decode attention */
+
+/* q [M, q_stride] fp32 (head h at columns [h d, h d + d)); k, v bf16 [n_heads][L_max][d];
+ * out [M, n_heads d] double. */
+void aio_oracle_attention(const float* q, int64_t q_stride, const uint16_t* k, const uint16_t* v, int64_t n_heads,
+                          int64_t d, int64_t L_max, int64_t L, int64_t M, double* out) {
+#pragma omp parallel for schedule(static) collapse(2)
+    for (int64_t m = 0; m < M; ++m)
+        for (int64_t h = 0; h < n_heads; ++h) {
+#if AIO_ORACLE_MUTANT == 12   /* causal limit off by one: sees the next new token */
+            int64_t last = L - M + m + 1 < L ? L - M + m + 1 : L - 1;
+#else
+            int64_t last = L - M + m;
+#endif
+#if AIO_ORACLE_MUTANT == 11   /* no 1/sqrt(d) scale */
+            double scale = 1.0;
+#else
+            double scale = 1.0 / sqrt((double)d);
+#endif
+            const float* qm = q + m * q_stride + h * d;
+            double mx = -INFINITY;
+            for (int64_t j = 0; j <= last; ++j) {
+                const uint16_t* kj = k + (h * L_max + j) * d;
+                double s = 0.0;
+                for (int64_t e = 0; e < d; ++e) s += (double)qm[e] * aio_oracle_bf16_to_double(kj[e]);
+                s *= scale;
+                if (s > mx) mx = s;
+            }
+            double* o = out + m * n_heads * d + h * d;
+            for (int64_t e = 0; e < d; ++e) o[e] = 0.0;
+            double sum = 0.0;
+            for (int64_t j = 0; j <= last; ++j) {
+                const uint16_t* kj = k + (h * L_max + j) * d;
+                const uint16_t* vj = v + (h * L_max + j) * d;
+                double s = 0.0;
+                for (int64_t e = 0; e < d; ++e) s += (double)qm[e] * aio_oracle_bf16_to_double(kj[e]);
+                double p = exp(s * scale - mx);
+                sum += p;
+                for (int64_t e = 0; e < d; ++e) o[e] += p * aio_oracle_bf16_to_double(vj[e]);
+            }
+#if AIO_ORACLE_MUTANT == 13   /* not normalised */
+            (void)sum;
+#else
+            for (int64_t e = 0; e < d; ++e) o[e] /= sum;
+#endif
+        }
 }

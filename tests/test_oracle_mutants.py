@@ -4,7 +4,9 @@ Each mutant is the oracle C source compiled with AIO_ORACLE_MUTANT=k:
   1 dropped term, 2 transposed operand, 3 wrong sign, 4 wrong scale index,
   5 dequantized weight rounded to bf16 before the product, 6 lost code sign,
   7 bf16 rounding toward zero, 8 sign error in the logistic of silu,
-  9 RMSNorm mean over K - 1, 10 SwiGLU gate and up swapped.
+  9 RMSNorm mean over K - 1, 10 SwiGLU gate and up swapped,
+  11 attention without the 1/sqrt(d) scale, 12 causal limit off by one, 13 attention output not
+  normalised.
 """
 import math
 import struct
@@ -78,9 +80,36 @@ def chain_pins_hold(o: oracle.Oracle) -> bool:
     return True
 
 
+def attention_pins_hold(o: oracle.Oracle) -> bool:
+    """A few of tests/test_oracle_attention_pins.py's facts, evaluated on an arbitrary build."""
+    d, L = 16, 2
+    k = np.zeros((1, L, d), np.uint16)
+    k[0, 0, 0] = _bf16_int(1)
+    v = np.zeros((1, L, d), np.uint16)
+    v[0, 0, 0] = _bf16_int(1)
+    v[0, 1, 1] = _bf16_int(1)
+    q = np.zeros((1, d), np.float32)
+    q[0, 0] = np.float32(math.sqrt(d) * math.log(3))
+    out = o.attention(q, k, v, L)
+    w0 = 1 / (1 + math.exp(-float(q[0, 0]) / math.sqrt(d)))
+    if abs(out[0, 0] - w0) > 1e-15 or abs(out[0, 1] - (1 - w0)) > 1e-15:
+        return False
+    L, M = 4, 2
+    k = np.zeros((1, L, 4), np.uint16)
+    for j in range(L):
+        k[0, j, 0] = _bf16_int(j)
+    v = np.zeros((1, L, 4), np.uint16)
+    for j in range(L):
+        v[0, j, 0] = _bf16_int(j + 1)
+    q = np.zeros((M, 4), np.float32)
+    q[:, 0] = 1e5
+    out = o.attention(q, k, v, L)
+    return out[0, 0] == 3.0 and out[1, 0] == 4.0
+
+
 def test_shipped_oracle_passes_pins():
     o = oracle.Oracle(oracle.load())
-    assert pins_hold(o) and chain_pins_hold(o)
+    assert pins_hold(o) and chain_pins_hold(o) and attention_pins_hold(o)
 
 
 @pytest.mark.parametrize("mutant", [1, 2, 3, 4, 5, 6])
@@ -93,3 +122,9 @@ def test_mutant_is_caught(tmp_path, mutant):
 def test_chain_mutant_is_caught(tmp_path, mutant):
     path = ob.build(out=str(tmp_path / f"libaio_oracle_m{mutant}.so"), mutant=mutant)
     assert not chain_pins_hold(oracle.Oracle(oracle.load(path)))
+
+
+@pytest.mark.parametrize("mutant", [11, 12, 13])
+def test_attention_mutant_is_caught(tmp_path, mutant):
+    path = ob.build(out=str(tmp_path / f"libaio_oracle_m{mutant}.so"), mutant=mutant)
+    assert not attention_pins_hold(oracle.Oracle(oracle.load(path)))
