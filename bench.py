@@ -430,6 +430,8 @@ def run_ours(args, wl):
         pld_sweep(args, peak)
     if args.chain and rank == 0:
         chain_lines(args, peak)
+    if args.attention and rank == 0:
+        attention_lines(args, peak)
     if pg is not None:
         pg.destroy_process_group()
     return 0
@@ -509,6 +511,60 @@ def chain_lines(args, peak):
         dw.close()
 
 
+def attention_lines(args, peak):
+    """Decode attention over KV caches of the 7B-class shapes (32 heads x 128) at the paper's 2K and
+    32K contexts, M = 1 and 3 (PLD look-ahead L = 2): one call per layer, over enough distinct layer
+    caches (seeded bf16 N(0, 1)) that a step streams more than 1 GB, well above L2; a step's calls
+    are captured in one CUDA graph.  One JSON line per (context, M): KV bytes per step / time."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    n_heads, d = 32, 128
+    gen = torch.Generator(device="cuda").manual_seed(args.seed)
+    stream = torch.cuda.Stream()
+    for L, layers in ((2048, 32), (32768, 4)):
+        caches = [(torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16),
+                   torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16)) for _ in range(layers)]
+        for M in (1, 3):
+            q = torch.randn(M, n_heads * d, device="cuda", generator=gen)
+            out = torch.empty(M, n_heads * d, device="cuda")
+            wsb = aio.aio_attention_workspace_bytes(M)
+            ws = torch.zeros(wsb, dtype=torch.uint8, device="cuda")
+
+            def step():
+                for kc, vc in caches:
+                    aio.aio_attention_decode(q.data_ptr(), n_heads * d, kc.data_ptr(), vc.data_ptr(), n_heads, d, L, L, M,
+                                             out.data_ptr(), ws.data_ptr(), wsb, stream.cuda_stream)
+            torch.cuda.synchronize()
+            for _ in range(args.warmup):
+                step()
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()            # one replay per step: no host gaps between layers
+            with torch.cuda.graph(graph, stream=stream):
+                step()
+            torch.cuda.synchronize()
+            for _ in range(args.warmup):
+                graph.replay()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            with torch.cuda.stream(stream):
+                for _ in range(args.steps):
+                    graph.replay()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            assert aio.aio_attention_check(ws.data_ptr()) == 0
+            ms = e0.elapsed_time(e1) / args.steps
+            kv_bytes = layers * 2 * n_heads * L * d * 2
+            gbs = kv_bytes / (ms / 1e3) / 1e9
+            print(json.dumps({"sweep": "attention", "workload": f"7b-attention-L{L}-M{M}", "L": L, "M": M,
+                              "layers": layers, "ms_per_step": round(ms, 4), "ms_per_layer": round(ms / layers, 5),
+                              "kv_bytes_per_step": kv_bytes, "value": round(gbs, 2), "unit": "GB/s",
+                              "frac_of_measured_peak": round(gbs / peak, 4), "launches_per_layer": 2,
+                              "steps": args.steps, "warmup": args.warmup}), flush=True)
+        del caches
+        torch.cuda.empty_cache()
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -525,6 +581,8 @@ def main():
                     help="after the main line, one line per PLD width M in {1,2,4,8} for bf16 and int8 7B steps")
     ap.add_argument("--chain", action="store_true",
                     help="after the main line, the chained 7B decoder step (x computed on the device), bf16 and int8")
+    ap.add_argument("--attention", action="store_true",
+                    help="after the main line, decode attention over 7B-shaped KV caches at 2K and 32K contexts")
     ap.add_argument("--step-mode", choices=["persistent", "chain"], default="persistent",
                     help="one cooperative launch per step (default) or one launch per projection")
     args = ap.parse_args()

@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 2
+#define AIO_ABI_VERSION 3
 
 typedef enum {
     AIO_OK = 0,
@@ -264,6 +264,32 @@ aio_status aio_decode_step_check(aio_step_t step, int* device_error);
 
 /* Free the step, its graph and its workspace (synchronises the device). NULL is accepted. */
 aio_status aio_decode_step_destroy(aio_step_t step);
+
+/*
+ * Decode attention over a KV cache (the long-context path the paper routes on: standard contexts
+ * up to 2K tokens, long ones up to 32K, Sec. 3.3 and Sec. 5.1).  M new tokens sit at positions
+ * L - M .. L - 1 of a cache holding L positions; token m attends to positions j <= L - M + m:
+ *   out[m, h*128 + e] = sum_j softmax_j(q[m, h] . k[h, j] / sqrt(128)) v[h, j, e].
+ * q:        fp32 [M, q_stride] (head h at columns [128 h, 128 h + 128)), device.
+ * k_cache,
+ * v_cache:  bf16 [n_heads][L_max][128], device (a run of positions of one head is contiguous).
+ * out:      fp32 [M, n_heads * 128], device.
+ * workspace: device scratch of aio_attention_workspace_bytes(M) bytes; its first 4 bytes are the
+ *           device error word and must be zero before the first call (aio_attention_check
+ *           clears it after reporting an error).  Calls sharing a workspace must not overlap.
+ * Arithmetic is fp32 with an online softmax; the per-warp partial results are merged in a fixed
+ * order, so results are reproducible.  Asynchronous on stream, allocates nothing.  Errors:
+ * INVALID_ARG (NULL pointer, M outside [1, 8], L outside [M, L_max], q_stride < 128 n_heads,
+ * workspace too small), UNSUPPORTED (head_dim != 128, n_heads above the grid's warp count),
+ * ALIGNMENT (a pointer not 16-byte aligned, q_stride not a multiple of 4), CUDA.
+ */
+aio_status aio_attention_workspace_bytes(int M, size_t* bytes);
+aio_status aio_attention_decode(const float* q, int q_stride, const void* k_cache, const void* v_cache, int n_heads,
+                                int head_dim, int L_max, int L, int M, float* out, void* workspace,
+                                size_t workspace_bytes, void* stream);
+
+/* Synchronise the device, then report (and clear) the attention workspace's device error word. */
+aio_status aio_attention_check(void* workspace, int* device_error);
 
 /*
  * Read-bandwidth probe: streams `bytes` from buf (device, 16-byte aligned, bytes a multiple of

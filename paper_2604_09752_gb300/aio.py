@@ -42,7 +42,7 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
-AIO_ABI_VERSION = 2
+AIO_ABI_VERSION = 3
 AIO_X_GIVEN = 0
 AIO_X_RMSNORM = 1
 AIO_X_SWIGLU = 2
@@ -97,6 +97,9 @@ _SIGS = {
     "aio_decode_step_reset": (_int, [_vp]),
     "aio_decode_step_destroy": (_int, [_vp]),
     "aio_probe_read": (_int, [_vp, _sz, _vp, _vp]),
+    "aio_attention_workspace_bytes": (_int, [_int, ctypes.POINTER(_sz)]),
+    "aio_attention_decode": (_int, [_vp, _int, _vp, _vp, _int, _int, _int, _int, _int, _vp, _vp, _sz, _vp]),
+    "aio_attention_check": (_int, [_vp, ctypes.POINTER(_int)]),
 }
 for _f, (_res, _args) in _SIGS.items():
     _fn = getattr(_lib, _f)
@@ -222,3 +225,21 @@ def aio_decode_step_destroy(step: int):
 
 def aio_probe_read(buf: int, nbytes: int, out: int, stream: int = 0):
     _check(_lib.aio_probe_read(buf, nbytes, out, stream), "aio_probe_read")
+
+
+def aio_attention_workspace_bytes(M: int) -> int:
+    b = _sz()
+    _check(_lib.aio_attention_workspace_bytes(M, ctypes.byref(b)), "aio_attention_workspace_bytes")
+    return b.value
+
+
+def aio_attention_decode(q: int, q_stride: int, k_cache: int, v_cache: int, n_heads: int, head_dim: int, L_max: int,
+                         L: int, M: int, out: int, workspace: int, workspace_bytes: int, stream: int = 0):
+    _check(_lib.aio_attention_decode(q, q_stride, k_cache, v_cache, n_heads, head_dim, L_max, L, M, out, workspace,
+                                     workspace_bytes, stream), "aio_attention_decode")
+
+
+def aio_attention_check(workspace: int) -> int:
+    e = _int()
+    _check(_lib.aio_attention_check(workspace, ctypes.byref(e)), "aio_attention_check")
+    return e.value

@@ -731,3 +731,55 @@ extern "C" aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N,
     AIO_CUDA(aio::launch_stream(a, wt == AIO_W_INT8_PERCHANNEL, geo.grid, s, !(flags & AIO_FLAG_NO_PDL), false));
     return AIO_OK;
 }
+
+// ------------------------------------------------------------------ decode attention
+extern "C" aio_status aio_attention_workspace_bytes(int M, size_t* bytes) {
+    if (!bytes) return fail(AIO_ERR_INVALID_ARG, "bytes is NULL");
+    if (M < 1 || M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, 8]", M);
+    int dev = -1, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    *bytes = aio::attn_workspace_bytes(sms * aio::kWarps, M);
+    return AIO_OK;
+}
+
+extern "C" aio_status aio_attention_decode(const float* q, int q_stride, const void* k_cache, const void* v_cache,
+                                           int n_heads, int head_dim, int L_max, int L, int M, float* out,
+                                           void* workspace, size_t workspace_bytes, void* stream) {
+    if (!q || !k_cache || !v_cache || !out || !workspace)
+        return fail(AIO_ERR_INVALID_ARG, "q, k_cache, v_cache, out and workspace must be non-NULL");
+    if (head_dim != 128) return fail(AIO_ERR_UNSUPPORTED, "head_dim=%d: only 128 is supported", head_dim);
+    if (M < 1 || M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, 8]", M);
+    if (n_heads < 1 || L < M || L > L_max)
+        return fail(AIO_ERR_INVALID_ARG, "need n_heads >= 1 and M <= L <= L_max (n_heads=%d M=%d L=%d L_max=%d)",
+                    n_heads, M, L, L_max);
+    if (q_stride < n_heads * 128) return fail(AIO_ERR_INVALID_ARG, "q_stride=%d < n_heads * 128", q_stride);
+    const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k_cache) |
+                          reinterpret_cast<uintptr_t>(v_cache) | reinterpret_cast<uintptr_t>(out) |
+                          reinterpret_cast<uintptr_t>(workspace);
+    if ((mis & 15u) || q_stride % 4 != 0)
+        return fail(AIO_ERR_ALIGNMENT, "q, the caches, out and workspace must be 16-byte aligned, q_stride a multiple of 4");
+    int dev = -1, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    if (n_heads > sms * aio::kWarps)
+        return fail(AIO_ERR_UNSUPPORTED, "n_heads=%d above %d (warps in the grid)", n_heads, sms * aio::kWarps);
+    const size_t need = aio::attn_workspace_bytes(sms * aio::kWarps, M);
+    if (workspace_bytes < need) return fail(AIO_ERR_INVALID_ARG, "workspace of %zu bytes, %zu needed", workspace_bytes, need);
+    AIO_CUDA(aio::launch_attention(q, q_stride, k_cache, v_cache, n_heads, L_max, L, M, out, workspace, sms,
+                                   kWaitLimitNs, static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}
+
+extern "C" aio_status aio_attention_check(void* workspace, int* device_error) {
+    if (!workspace) return fail(AIO_ERR_INVALID_ARG, "workspace is NULL");
+    int dev = -1;
+    AIO_CUDA(cudaGetDevice(&dev));
+    AIO_CUDA(cudaDeviceSynchronize());
+    int e = 0;
+    AIO_CUDA(cudaMemcpy(&e, workspace, sizeof e, cudaMemcpyDeviceToHost));
+    if (e) AIO_CUDA(cudaMemset(workspace, 0, sizeof e));
+    if (device_error) *device_error = e;
+    if (e) return fail(AIO_ERR_DEVICE_TIMEOUT, "a bounded device wait expired (code %d)", e);
+    return AIO_OK;
+}

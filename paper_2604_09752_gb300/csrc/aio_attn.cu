@@ -1,0 +1,355 @@
+// aio_attn.cu -- decode attention over a KV cache: the long-context half of the paper's routing
+// (contexts up to 2K tokens are standard, up to 32K long: Sec. 3.3, Sec. 5.1).  For M new tokens
+// at positions L - M .. L - 1 of a cache of L positions, per head h of dimension 128:
+//   s_j = q[m, h] . k[h, j] / sqrt(128)   for j <= L - M + m,   out[m, h] = sum_j softmax(s)_j v[h, j].
+//
+// Like the projections, this streams bytes from HBM (2 * 256 B per position and head) with a few
+// flops per byte, so it reuses the stream kernel's machinery: one CTA of 8 warps per SM, a ring of
+// bulk copies per warp, and an even split of the work over all warps.
+//   * Cache layout: [head][position][128] bf16, so a run of positions of one head is contiguous.
+//   * Units: 16 positions of one head (4 KB of K and 4 KB of V, one ring slot).  The n_heads *
+//     ceil(L / 16) units, head-major, are split evenly over the Z warps.  A warp's units span at
+//     most two heads (n_heads <= Z), so it produces at most two partial results.
+//   * Per unit: lane l holds dims [4l, 4l + 4) of q (fp32, scaled by log2(e) / sqrt(128)) for every
+//     token.  The 16 partial dot products of a lane are reduced across the warp with 16 shuffles
+//     (a transposing reduction: each halving step trades the half of the values a lane does not
+//     keep), then the lane pair 2p, 2p + 1 holds position p's score.  An online softmax in base 2
+//     keeps a running max, sum and weighted sum of V (lane l: dims [4l, 4l + 4)).
+//   * A second small kernel merges each head's partials (max, sum, weighted V) in a fixed order, so
+//     the result does not depend on timing.
+#include "aio_stream.cuh"
+
+namespace aio {
+namespace {
+
+constexpr int kHeadDim = 128;
+constexpr int kAttnPos = 16;                                  // positions per unit
+constexpr int kAttnUnitBytes = kAttnPos * kHeadDim * 2;       // 4 KB of K (and of V) per unit
+constexpr int kAttnSlot = 2 * kAttnUnitBytes;                 // K then V
+constexpr int kAttnStages = kRingBytesPerWarp / kAttnSlot;    // 3 slots of 8 KB per warp
+constexpr int kAttnSmem = kWarps * kAttnStages * kAttnSlot + kWarps * kAttnStages * 8;
+constexpr int kAttnRec = 132;                                 // floats per partial: 128 weighted V, max, sum, pad
+static_assert(kAttnStages >= 2, "attention ring");
+
+struct AttnArgs {
+    const float* q;           // [M, q_stride]
+    const uint16_t* k;        // [n_heads][L_max][128]
+    const uint16_t* v;
+    float* out;               // [M, n_heads * 128]
+    float* part;              // [Z][2][M][kAttnRec]
+    int* err;
+    int q_stride, n_heads, L_max, L, M, Z, nch;
+    long long U;              // units = n_heads * nch
+    unsigned long long wait_limit_ns;
+};
+
+__device__ __forceinline__ long long attn_seg(long long z, long long U, int Z) { return z * U / Z; }
+
+__device__ __forceinline__ uint2 lds64(uint32_t addr) {
+    uint2 v;
+    asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+// Sum over the warp of 16 per-lane values a[0..15] (one per position); returns, in lane l, the
+// total for position (l >> 1) & 15.  Each step halves the values a lane holds: lanes whose bit o is
+// set keep the upper half and send the lower, the others the reverse, so 8 + 4 + 2 + 1 + 1 shuffles
+// replace 16 separate 5-step butterflies.
+__device__ __forceinline__ float warp_sum16_transpose(float (&a)[16], int lane) {
+#pragma unroll
+    for (int o = 16, n = 8; o >= 2; o >>= 1, n >>= 1) {
+        const bool hi = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < n; ++i) {
+            const float send = hi ? a[i] : a[i + n];
+            const float keep = hi ? a[i + n] : a[i];
+            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    return a[0] + __shfl_xor_sync(0xffffffffu, a[0], 1);
+}
+
+template <int MT>
+__global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __grid_constant__ AttnArgs a) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint8_t* ring = smem + warp * kAttnStages * kAttnSlot;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kAttnStages * kAttnSlot) + warp * kAttnStages;
+    const long long z = static_cast<long long>(blockIdx.x) * kWarps + warp;
+    if (lane == 0) {
+#pragma unroll
+        for (int i = 0; i < kAttnStages; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+    const long long u0 = attn_seg(z, a.U, a.Z), u1 = attn_seg(z + 1, a.U, a.Z);
+    const uint64_t pol = policy_evict_first();
+
+    // issue side: unit u -> head u / nch, positions [16 (u % nch), +16) clipped to L; the head and
+    // chunk are tracked incrementally (one division per warp)
+    long long ui = u0;
+    int ih = static_cast<int>(u0 / a.nch), ic = static_cast<int>(u0 - static_cast<long long>(ih) * a.nch);
+    auto issue = [&](int slot) {
+        if (ui >= u1) return;
+        const int h = ih, c = ic;
+        if (++ic == a.nch) {
+            ic = 0;
+            ++ih;
+        }
+        const int p0 = c * kAttnPos, np = min(kAttnPos, a.L - p0);
+        const uint32_t bytes = static_cast<uint32_t>(np * kHeadDim * 2);
+        const size_t off = (static_cast<size_t>(h) * a.L_max + p0) * kHeadDim;
+        if (lane == 0) {
+            mbar_expect_tx(&bars[slot], 2 * bytes);
+            bulk_g2s(ring + slot * kAttnSlot, a.k + off, bytes, &bars[slot], pol);
+            bulk_g2s(ring + slot * kAttnSlot + kAttnUnitBytes, a.v + off, bytes, &bars[slot], pol);
+        }
+        ++ui;
+    };
+    int in_flight = 0;
+    for (int i = 0; i < kAttnStages && ui < u1; ++i) {
+        issue(i);
+        ++in_flight;
+    }
+
+    const float qscale = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));   // log2(e) / sqrt(d)
+    float4 q4[MT];
+    float mx[MT], ls[MT];
+    float4 acc[MT];
+    int head = -1, seg_idx = -1;
+    bool dead = false;
+    auto flush = [&]() {   // this warp's partial for `head` into record seg_idx
+        if (head < 0) return;
+        float* base = a.part + (static_cast<size_t>(z) * 2 + seg_idx) * a.M * kAttnRec;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            float* r = base + m * kAttnRec;
+            *reinterpret_cast<float4*>(r + 4 * lane) = acc[m];
+            if (lane == 0) {
+                r[128] = mx[m];
+                r[129] = ls[m];
+            }
+        }
+    };
+    int cslot = 0;
+    uint32_t cphase = 0;
+    int h = static_cast<int>(u0 / a.nch), c = static_cast<int>(u0 - static_cast<long long>(h) * a.nch) - 1;
+    for (long long u = u0; u < u1; ++u) {
+        if (++c == a.nch) {
+            c = 0;
+            ++h;
+        }
+        if (h != head) {
+            flush();
+            head = h;
+            ++seg_idx;
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+                const float4 t = *reinterpret_cast<const float4*>(a.q + static_cast<size_t>(m) * a.q_stride + h * kHeadDim + 4 * lane);
+                q4[m] = make_float4(t.x * qscale, t.y * qscale, t.z * qscale, t.w * qscale);
+                mx[m] = -INFINITY;
+                ls[m] = 0.0f;
+                acc[m] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            }
+        }
+        if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, a.wait_limit_ns))) {
+            if (lane == 0) atomicCAS(a.err, 0, kDevErrTimeout);
+            dead = true;   // cslot is the slot that timed out; in_flight counts it
+            break;
+        }
+        {
+            const int p0 = c * kAttnPos, np = min(kAttnPos, a.L - p0);
+            const uint32_t kaddr = smem_addr(ring + cslot * kAttnSlot) + 8 * lane;
+            const uint32_t vaddr = kaddr + kAttnUnitBytes;
+            uint2 kr[kAttnPos];
+#pragma unroll
+            for (int j = 0; j < kAttnPos; ++j) kr[j] = j < np ? lds64(kaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+                float part[kAttnPos];
+#pragma unroll
+                for (int j = 0; j < kAttnPos; ++j) {
+                    const float k0 = __uint_as_float(kr[j].x << 16), k1 = __uint_as_float(kr[j].x & 0xFFFF0000u);
+                    const float k2 = __uint_as_float(kr[j].y << 16), k3 = __uint_as_float(kr[j].y & 0xFFFF0000u);
+                    part[j] = fmaf(q4[m].w, k3, fmaf(q4[m].z, k2, fmaf(q4[m].y, k1, q4[m].x * k0)));
+                }
+                // lanes 2p and 2p + 1 hold position p's score (base-2 logits)
+                const int pos = (lane >> 1) & 15;
+                float s = warp_sum16_transpose(part, lane);
+                const bool visible = pos < np && p0 + pos <= a.L - a.M + m;
+                s = visible ? s : -INFINITY;
+                float bm = s;
+#pragma unroll
+                for (int o = 2; o < 32; o <<= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
+                const float nm = fmaxf(mx[m], bm);
+                if (nm != -INFINITY) {
+                    const float alpha = exp2f(mx[m] - nm);   // 0 while mx is -inf
+                    const float p = visible ? exp2f(s - nm) : 0.0f;
+                    float psum = p;
+#pragma unroll
+                    for (int o = 2; o < 32; o <<= 1) psum += __shfl_xor_sync(0xffffffffu, psum, o);
+                    ls[m] = ls[m] * alpha + psum;
+                    float4 ac = make_float4(acc[m].x * alpha, acc[m].y * alpha, acc[m].z * alpha, acc[m].w * alpha);
+#pragma unroll
+                    for (int j = 0; j < kAttnPos; ++j) {
+                        const float pj = __shfl_sync(0xffffffffu, p, 2 * j);
+                        if (j < np) {
+                            const uint2 vr = lds64(vaddr + j * (kHeadDim * 2));
+                            ac.x = fmaf(pj, __uint_as_float(vr.x << 16), ac.x);
+                            ac.y = fmaf(pj, __uint_as_float(vr.x & 0xFFFF0000u), ac.y);
+                            ac.z = fmaf(pj, __uint_as_float(vr.y << 16), ac.z);
+                            ac.w = fmaf(pj, __uint_as_float(vr.y & 0xFFFF0000u), ac.w);
+                        }
+                    }
+                    acc[m] = ac;
+                    mx[m] = nm;
+                }
+            }
+        }
+        __syncwarp();   // every lane's reads of the slot are done before it is refilled
+        const int done_slot = cslot;
+        cslot = (cslot + 1 == kAttnStages) ? 0 : cslot + 1;
+        cphase ^= (cslot == 0) ? 1u : 0u;
+        if (ui < u1) {
+            issue(done_slot);
+        } else {
+            --in_flight;
+        }
+    }
+    if (dead) {   // wait (bounded) for this warp's copies still in flight, then leave
+        for (int j = 0; j < in_flight; ++j) {
+            mbar_wait(&bars[cslot], cphase, a.wait_limit_ns);
+            cslot = (cslot + 1 == kAttnStages) ? 0 : cslot + 1;
+            cphase ^= (cslot == 0) ? 1u : 0u;
+        }
+    }
+    flush();
+}
+
+// One CTA per (head, token): merges the partials of the warps whose units cover the head.  Every
+// warp reduces the partials' maxima (lane i: the i-th covering warp, 32 at a time) to the global
+// max; warp w then adds the weighted sums and weighted V vectors of partials w, w + 8, ... (lane l:
+// dims [4l, 4l + 4)), and warp 0 adds the 8 warps' results in order: a fixed order, whatever the
+// timing.
+__global__ void __launch_bounds__(kThreads) aio_attn_combine_kernel(const __grid_constant__ AttnArgs a) {
+    __shared__ float4 wacc[kWarps][32];
+    __shared__ float wl[kWarps];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.x / a.M, m = blockIdx.x - h * a.M;
+    const long long ua = static_cast<long long>(h) * a.nch, ub = ua + a.nch - 1;   // the head's units
+    long long zlo = ua * a.Z / a.U;   // the warp holding unit ua
+    while (zlo > 0 && attn_seg(zlo, a.U, a.Z) > ua) --zlo;
+    while (attn_seg(zlo + 1, a.U, a.Z) <= ua) ++zlo;
+    long long zhi = ub * a.Z / a.U;   // the warp holding unit ub
+    while (zhi > 0 && attn_seg(zhi, a.U, a.Z) > ub) --zhi;
+    while (attn_seg(zhi + 1, a.U, a.Z) <= ub) ++zhi;
+    const int n = static_cast<int>(zhi - zlo + 1);
+    // record of covering warp i, or -1 for an empty segment
+    auto record = [&](int i) -> long long {
+        const long long zz = zlo + i;
+        const long long s0 = attn_seg(zz, a.U, a.Z);
+        if (attn_seg(zz + 1, a.U, a.Z) == s0) return -1;
+        const int si = s0 / a.nch == h ? 0 : 1;
+        return ((zz * 2 + si) * a.M + m) * kAttnRec;
+    };
+    float M_ = -INFINITY;
+    for (int b0 = 0; b0 < n; b0 += 32) {
+        float mx = -INFINITY;
+        if (b0 + lane < n) {
+            const long long r = record(b0 + lane);
+            if (r >= 0) mx = a.part[r + 128];
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        M_ = fmaxf(M_, mx);
+    }
+    float l = 0.0f;
+    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    for (int i = warp; i < n; i += kWarps) {
+        const long long r = record(i);
+        if (r < 0) continue;
+        const float pm = a.part[r + 128];
+        const float w = pm == -INFINITY ? 0.0f : exp2f(pm - M_);
+        l = fmaf(a.part[r + 129], w, l);
+        const float4 v = *reinterpret_cast<const float4*>(a.part + r + 4 * lane);
+        acc = make_float4(fmaf(v.x, w, acc.x), fmaf(v.y, w, acc.y), fmaf(v.z, w, acc.z), fmaf(v.w, w, acc.w));
+    }
+    wacc[warp][lane] = acc;
+    if (lane == 0) wl[warp] = l;
+    __syncthreads();
+    if (warp == 0) {
+        float lt = 0.0f;
+        float4 at = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) {
+            lt += wl[w];
+            const float4 v = wacc[w][lane];
+            at = make_float4(at.x + v.x, at.y + v.y, at.z + v.z, at.w + v.w);
+        }
+        const float inv = 1.0f / lt;
+        *reinterpret_cast<float4*>(a.out + static_cast<size_t>(m) * a.n_heads * kHeadDim + h * kHeadDim + 4 * lane) =
+            make_float4(at.x * inv, at.y * inv, at.z * inv, at.w * inv);
+    }
+}
+
+using AttnFn = void (*)(const AttnArgs);
+
+AttnFn attn_fn(int M) {
+    switch (M) {
+        case 1: return aio_attn_partial_kernel<1>;
+        case 2: return aio_attn_partial_kernel<2>;
+        case 3: return aio_attn_partial_kernel<3>;
+        case 4: return aio_attn_partial_kernel<4>;
+        case 5: return aio_attn_partial_kernel<5>;
+        case 6: return aio_attn_partial_kernel<6>;
+        case 7: return aio_attn_partial_kernel<7>;
+        case 8: return aio_attn_partial_kernel<8>;
+        default: return nullptr;
+    }
+}
+
+}  // namespace
+
+size_t attn_workspace_bytes(int Z, int M) {
+    return 256 + static_cast<size_t>(Z) * 2 * M * kAttnRec * sizeof(float);
+}
+
+cudaError_t launch_attention(const float* q, int q_stride, const void* k, const void* v, int n_heads, int L_max, int L,
+                             int M, float* out, void* ws, int grid, unsigned long long wait_limit_ns, cudaStream_t s) {
+    AttnFn f = attn_fn(M);
+    if (!f) return cudaErrorInvalidValue;
+    static thread_local int prepared_device = -1;
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (prepared_device != dev) {
+        for (int i = 1; i <= kMaxM; ++i) {
+            e = cudaFuncSetAttribute(attn_fn(i), cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+            if (e != cudaSuccess) return e;
+        }
+        prepared_device = dev;
+    }
+    AttnArgs a = {};
+    a.q = q;
+    a.k = static_cast<const uint16_t*>(k);
+    a.v = static_cast<const uint16_t*>(v);
+    a.out = out;
+    a.err = static_cast<int*>(ws);
+    a.part = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + 256);
+    a.q_stride = q_stride;
+    a.n_heads = n_heads;
+    a.L_max = L_max;
+    a.L = L;
+    a.M = M;
+    a.Z = grid * kWarps;
+    a.nch = (L + kAttnPos - 1) / kAttnPos;
+    a.U = static_cast<long long>(n_heads) * a.nch;
+    a.wait_limit_ns = wait_limit_ns;
+    f<<<grid, kThreads, kAttnSmem, s>>>(a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    aio_attn_combine_kernel<<<n_heads * M, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace aio
