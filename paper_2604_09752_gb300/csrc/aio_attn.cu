@@ -226,12 +226,16 @@ __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __g
     flush();
 }
 
-// One CTA per (head, token): merges the partials of the warps whose units cover the head.  Every
-// warp reduces the partials' maxima (lane i: the i-th covering warp, 32 at a time) to the global
-// max; warp w then adds the weighted sums and weighted V vectors of partials w, w + 8, ... (lane l:
-// dims [4l, 4l + 4)), and warp 0 adds the 8 warps' results in order: a fixed order, whatever the
-// timing.
+// One CTA per (head, token): merges the partials of the warps whose units cover the head.  The
+// threads first list the covering warps' records and maxima in shared memory (in parallel); each
+// warp then reduces the maxima to the global max, adds the weighted sums and weighted V vectors of
+// records w, w + 8, ... (lane l: dims [4l, 4l + 4)), and warp 0 adds the 8 warps' results in order:
+// a fixed order, whatever the timing.
+constexpr int kCombineMax = kAttnMaxWarps;   // covering warps listed in shared memory
+
 __global__ void __launch_bounds__(kThreads) aio_attn_combine_kernel(const __grid_constant__ AttnArgs a) {
+    __shared__ long long srec[kCombineMax];
+    __shared__ float smx[kCombineMax];
     __shared__ float4 wacc[kWarps][32];
     __shared__ float wl[kWarps];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -243,33 +247,32 @@ __global__ void __launch_bounds__(kThreads) aio_attn_combine_kernel(const __grid
     long long zhi = ub * a.Z / a.U;   // the warp holding unit ub
     while (zhi > 0 && attn_seg(zhi, a.U, a.Z) > ub) --zhi;
     while (attn_seg(zhi + 1, a.U, a.Z) <= ub) ++zhi;
-    const int n = static_cast<int>(zhi - zlo + 1);
-    // record of covering warp i, or -1 for an empty segment
-    auto record = [&](int i) -> long long {
+    const int n = min(static_cast<int>(zhi - zlo + 1), kCombineMax);
+    for (int i = threadIdx.x; i < n; i += kThreads) {
         const long long zz = zlo + i;
         const long long s0 = attn_seg(zz, a.U, a.Z);
-        if (attn_seg(zz + 1, a.U, a.Z) == s0) return -1;
-        const int si = s0 / a.nch == h ? 0 : 1;
-        return ((zz * 2 + si) * a.M + m) * kAttnRec;
-    };
-    float M_ = -INFINITY;
-    for (int b0 = 0; b0 < n; b0 += 32) {
+        long long r = -1;
         float mx = -INFINITY;
-        if (b0 + lane < n) {
-            const long long r = record(b0 + lane);
-            if (r >= 0) mx = a.part[r + 128];
+        if (attn_seg(zz + 1, a.U, a.Z) > s0) {   // non-empty segment
+            const int si = s0 / a.nch == h ? 0 : 1;
+            r = ((zz * 2 + si) * a.M + m) * kAttnRec;
+            mx = a.part[r + 128];
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        M_ = fmaxf(M_, mx);
+        srec[i] = r;
+        smx[i] = mx;
     }
+    __syncthreads();
+    float M_ = -INFINITY;
+    for (int i = lane; i < n; i += 32) M_ = fmaxf(M_, smx[i]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M_ = fmaxf(M_, __shfl_xor_sync(0xffffffffu, M_, o));
     float l = 0.0f;
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll 4
     for (int i = warp; i < n; i += kWarps) {
-        const long long r = record(i);
+        const long long r = srec[i];
         if (r < 0) continue;
-        const float pm = a.part[r + 128];
-        const float w = pm == -INFINITY ? 0.0f : exp2f(pm - M_);
+        const float w = smx[i] == -INFINITY ? 0.0f : exp2f(smx[i] - M_);
         l = fmaf(a.part[r + 129], w, l);
         const float4 v = *reinterpret_cast<const float4*>(a.part + r + 4 * lane);
         acc = make_float4(fmaf(v.x, w, acc.x), fmaf(v.y, w, acc.y), fmaf(v.z, w, acc.z), fmaf(v.w, w, acc.w));

@@ -26,6 +26,8 @@ def main():
     ap.add_argument("--layers", type=int, default=0, help="with --step: keep only this many layers (0 = all)")
     ap.add_argument("--mode", choices=["persistent", "chain"], default="persistent")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--attention", type=int, default=0, metavar="L",
+                    help="run decode attention over a 7B-shaped KV cache of L positions (32 heads x 128) instead")
     args = ap.parse_args()
 
     import torch
@@ -33,6 +35,8 @@ def main():
     from paper_2604_09752_gb300.workload import DeviceWorkload
     from synth import workloads as swl
 
+    if args.attention:
+        return attention_case(args)
     wl = swl.WORKLOADS[args.workload]
     if args.step:
         L = max(p.layer for p in wl.projs)
@@ -57,6 +61,36 @@ def main():
     gb = dw.weight_bytes() / 1e9
     print(f"{args.workload} {'step' if args.step else args.proj} M={args.M}: {ms:.4f} ms, {gb / ms * 1e3:.1f} GB/s")
     dw.close()
+
+
+def attention_case(args):
+    """One layer's decode attention (32 heads x 128, seeded bf16 N(0, 1) caches), reps calls."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    n_heads, d, L, M = 32, 128, args.attention, args.M
+    gen = torch.Generator(device="cuda").manual_seed(0)
+    k = torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16)
+    v = torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16)
+    q = torch.randn(M, n_heads * d, device="cuda", generator=gen)
+    out = torch.empty(M, n_heads * d, device="cuda")
+    wsb = aio.aio_attention_workspace_bytes(M)
+    ws = torch.zeros(wsb, dtype=torch.uint8, device="cuda")
+
+    def run():
+        aio.aio_attention_decode(q.data_ptr(), n_heads * d, k.data_ptr(), v.data_ptr(), n_heads, d, L, L, M, out.data_ptr(),
+                                 ws.data_ptr(), wsb, torch.cuda.current_stream().cuda_stream)
+    run()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.reps):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    assert aio.aio_attention_check(ws.data_ptr()) == 0
+    ms = e0.elapsed_time(e1) / args.reps
+    kv = 2 * n_heads * L * d * 2
+    print(f"attention L={L} M={M}: {ms:.4f} ms per call, {kv / ms / 1e6:.1f} GB/s of KV")
 
 
 if __name__ == "__main__":
