@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "aio.h"
+#include "aio_attn.h"
 #include "aio_internal.h"
 
 namespace {

@@ -17,6 +17,7 @@
 //     keeps a running max, sum and weighted sum of V (lane l: dims [4l, 4l + 4)).
 //   * A second small kernel merges each head's partials (max, sum, weighted V) in a fixed order, so
 //     the result does not depend on timing.
+#include "aio_attn.h"
 #include "aio_stream.cuh"
 
 namespace aio {

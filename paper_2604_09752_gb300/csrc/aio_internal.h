@@ -130,11 +130,6 @@ StreamFn chain_stream_fn(bool i8, int M);   // aio_chain.cu
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop,
                           bool chained = false);
 cudaError_t occupancy(bool i8, int M, bool chained, int* blocks_per_sm);
-// Decode attention (aio_attn.cu): workspace bytes for Z warps and M tokens, and the two launches.
-constexpr int kAttnMaxWarps = 1536;   // warps in the grid the merge kernel can list (host-checked)
-size_t attn_workspace_bytes(int Z, int M);
-cudaError_t launch_attention(const float* q, int q_stride, const void* k, const void* v, int n_heads, int L_max, int L,
-                             int M, float* out, void* ws, int grid, unsigned long long wait_limit_ns, cudaStream_t s);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
 cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s);
 
