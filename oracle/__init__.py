@@ -19,6 +19,9 @@ Functions and the passages they follow:
   * double_to_bf16(v)        round a double to bf16, nearest-even.
   * attention(q, k, v, L)    decode attention of M new tokens over a KV cache of
                              L positions (the long-context path, Sec. 3.3, Sec. 5.1).
+  * pld.draft / pld.argmax / pld.accept  prompt-lookup drafting (N = 6, L = 2,
+                             Sec. 4.2) and greedy acceptance of the verification
+                             pass (oracle/pld.py, plain Python).
   * silu(t), rmsnorm(...), swiglu(...), slice_x(...)
                              the steps between the projections of a chained
                              decoder step; chain_step(...) runs a whole chained
@@ -32,7 +35,8 @@ Parity status: every function above is pinned by tests/test_oracle_pins.py
 (brute force, one-hot, identity/zero, linearity, exact dequant, fp64 error
 bound against exact rational sums), tests/test_oracle_chain_pins.py (bf16
 rounding against exact rationals and a library conversion, closed forms of the
-logistic, RMSNorm invariants, exact residual adds) and
+logistic, RMSNorm invariants, exact residual adds),
+tests/test_oracle_attention_pins.py, tests/test_oracle_pld_pins.py and
 tests/test_oracle_mutants.py.
 """
 from __future__ import annotations
