@@ -428,6 +428,7 @@ def run_ours(args, wl):
     dw.close()
     if args.pld_sweep and rank == 0:
         pld_sweep(args, peak)
+        pld_ops_line(args)
     if args.chain and rank == 0:
         chain_lines(args, peak)
     if args.attention and rank == 0:
@@ -473,6 +474,46 @@ def pld_sweep(args, peak):
                               "verified_tokens_per_s_upper_bound": round(1000.0 * M / ms, 2),
                               "steps": args.steps, "warmup": args.warmup}), flush=True)
         dw.close()
+
+
+def pld_ops_line(args):
+    """Latency of the work around a PLD verification pass (Sec. 4.2, N = 6, L = 2): drafting over a
+    2K and a 32K token history, the argmax of 3 rows of 32000 logits, and the acceptance check;
+    each captured in a CUDA graph and replayed, so the figure is device time per call."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    gen = torch.Generator(device="cuda").manual_seed(args.seed)
+    stream = torch.cuda.Stream()
+    res = {}
+    for name, T in (("draft_2k", 2048), ("draft_32k", 32768)):
+        toks = torch.randint(0, 32000, (T,), dtype=torch.int32, device="cuda", generator=gen)
+        out = torch.zeros(5, dtype=torch.int32, device="cuda")
+        res[name] = (lambda t=toks, o=out, n=T: aio.aio_pld_draft(t.data_ptr(), n, 6, 2, o.data_ptr(), stream.cuda_stream))
+    logits = torch.randn(3, 32000, device="cuda", generator=gen)
+    am = torch.zeros(3, dtype=torch.int32, device="cuda")
+    res["argmax_3x32000"] = lambda: aio.aio_argmax_rows(logits.data_ptr(), 3, 32000, 32000, am.data_ptr(), stream.cuda_stream)
+    dbuf = torch.tensor([2, 2, 0, 1, 2], dtype=torch.int32, device="cuda")
+    acc = torch.zeros(2, dtype=torch.int32, device="cuda")
+    res["accept"] = lambda: aio.aio_pld_accept(am.data_ptr(), dbuf.data_ptr(), acc.data_ptr(), stream.cuda_stream)
+    line = {"sweep": "pld_ops", "unit": "us per call"}
+    for name, fn in res.items():
+        reps = 50
+        fn()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        line[name] = round(e0.elapsed_time(e1) * 1e3 / reps, 2)
+    print(json.dumps(line), flush=True)
 
 
 def chain_lines(args, peak):

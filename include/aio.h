@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 3
+#define AIO_ABI_VERSION 4
 
 typedef enum {
     AIO_OK = 0,
@@ -290,6 +290,32 @@ aio_status aio_attention_decode(const float* q, int q_stride, const void* k_cach
 
 /* Synchronise the device, then report (and clear) the attention workspace's device error word. */
 aio_status aio_attention_check(void* workspace, int* device_error);
+
+/*
+ * Prompt-lookup decoding around the verification pass (Sec. 4.2: n-gram window N = 6, look-ahead
+ * L = 2).  All device pointers, asynchronous on stream, no allocation; the paper prints no
+ * algorithm, so these state the reading.
+ *
+ * aio_pld_draft: tokens [T] int32.  Among positions i < T - 1, the one whose preceding tokens
+ * share the longest suffix (n <= N tokens) with the whole sequence, the most recent among equals;
+ * the draft is the up to L tokens after it (fewer at the end of the sequence, none without a
+ * match).  out [3 + L] int32: draft length d, matched n, position i (-1 without a match), then the
+ * d drafted tokens (-1 after them).  1 <= N <= 32, 1 <= L <= 7.
+ *
+ * aio_argmax_rows: out[m] = argmax over v < V of logits[m * stride + v] (fp32), the lowest index
+ * among equal maxima; a NaN counts as the maximum (the first NaN wins).  1 <= M <= 65535.
+ *
+ * aio_pld_accept: greedy acceptance.  argmax [d + 1] holds the verification pass's argmax for the
+ * last committed token followed by the d drafted tokens; draft is aio_pld_draft's out.  result [2]
+ * int32: the number a of drafted tokens accepted (the longest agreeing prefix), then the model's
+ * next token argmax[a]: a + 1 tokens commit.
+ *
+ * Errors: INVALID_ARG (NULL pointer, a size outside its range), ALIGNMENT (a pointer not 4-byte
+ * aligned), UNSUPPORTED (not a GB300), CUDA.
+ */
+aio_status aio_pld_draft(const int* tokens, int T, int N, int L, int* out, void* stream);
+aio_status aio_argmax_rows(const float* logits, int M, int V, int stride, int* out, void* stream);
+aio_status aio_pld_accept(const int* argmax, const int* draft, int* result, void* stream);
 
 /*
  * Read-bandwidth probe: streams `bytes` from buf (device, 16-byte aligned, bytes a multiple of

@@ -42,7 +42,7 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
-AIO_ABI_VERSION = 3
+AIO_ABI_VERSION = 4
 AIO_X_GIVEN = 0
 AIO_X_RMSNORM = 1
 AIO_X_SWIGLU = 2
@@ -100,6 +100,9 @@ _SIGS = {
     "aio_attention_workspace_bytes": (_int, [_int, ctypes.POINTER(_sz)]),
     "aio_attention_decode": (_int, [_vp, _int, _vp, _vp, _int, _int, _int, _int, _int, _vp, _vp, _sz, _vp]),
     "aio_attention_check": (_int, [_vp, ctypes.POINTER(_int)]),
+    "aio_pld_draft": (_int, [_vp, _int, _int, _int, _vp, _vp]),
+    "aio_argmax_rows": (_int, [_vp, _int, _int, _int, _vp, _vp]),
+    "aio_pld_accept": (_int, [_vp, _vp, _vp, _vp]),
 }
 for _f, (_res, _args) in _SIGS.items():
     _fn = getattr(_lib, _f)
@@ -243,3 +246,15 @@ def aio_attention_check(workspace: int) -> int:
     e = _int()
     _check(_lib.aio_attention_check(workspace, ctypes.byref(e)), "aio_attention_check")
     return e.value
+
+
+def aio_pld_draft(tokens: int, T: int, N: int, L: int, out: int, stream: int = 0):
+    _check(_lib.aio_pld_draft(tokens, T, N, L, out, stream), "aio_pld_draft")
+
+
+def aio_argmax_rows(logits: int, M: int, V: int, stride: int, out: int, stream: int = 0):
+    _check(_lib.aio_argmax_rows(logits, M, V, stride, out, stream), "aio_argmax_rows")
+
+
+def aio_pld_accept(argmax: int, draft: int, result: int, stream: int = 0):
+    _check(_lib.aio_pld_accept(argmax, draft, result, stream), "aio_pld_accept")

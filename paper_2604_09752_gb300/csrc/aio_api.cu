@@ -15,6 +15,7 @@
 
 #include "aio.h"
 #include "aio_attn.h"
+#include "aio_pld.h"
 #include "aio_internal.h"
 
 namespace {
@@ -784,5 +785,44 @@ extern "C" aio_status aio_attention_check(void* workspace, int* device_error) {
     if (e) AIO_CUDA(cudaMemset(workspace, 0, sizeof e));
     if (device_error) *device_error = e;
     if (e) return fail(AIO_ERR_DEVICE_TIMEOUT, "a bounded device wait expired (code %d)", e);
+    return AIO_OK;
+}
+
+// ------------------------------------------------------------------ prompt-lookup decoding
+extern "C" aio_status aio_pld_draft(const int* tokens, int T, int N, int L, int* out, void* stream) {
+    if (!tokens || !out) return fail(AIO_ERR_INVALID_ARG, "tokens and out must be non-NULL");
+    if (T < 1 || N < 1 || N > aio::kPldMaxN || L < 1 || L > aio::kPldMaxL)
+        return fail(AIO_ERR_INVALID_ARG, "need T >= 1, 1 <= N <= %d, 1 <= L <= %d (T=%d N=%d L=%d)", aio::kPldMaxN,
+                    aio::kPldMaxL, T, N, L);
+    if ((reinterpret_cast<uintptr_t>(tokens) | reinterpret_cast<uintptr_t>(out)) & 3u)
+        return fail(AIO_ERR_ALIGNMENT, "tokens and out must be 4-byte aligned");
+    int dev = -1, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    AIO_CUDA(aio::launch_pld_draft(tokens, T, N, L, out, static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}
+
+extern "C" aio_status aio_argmax_rows(const float* logits, int M, int V, int stride, int* out, void* stream) {
+    if (!logits || !out) return fail(AIO_ERR_INVALID_ARG, "logits and out must be non-NULL");
+    if (M < 1 || M > 65535 || V < 1 || stride < V)
+        return fail(AIO_ERR_INVALID_ARG, "need 1 <= M <= 65535, V >= 1, stride >= V (M=%d V=%d stride=%d)", M, V, stride);
+    if ((reinterpret_cast<uintptr_t>(logits) | reinterpret_cast<uintptr_t>(out)) & 3u)
+        return fail(AIO_ERR_ALIGNMENT, "logits and out must be 4-byte aligned");
+    int dev = -1, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    AIO_CUDA(aio::launch_argmax(logits, M, V, stride, out, static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}
+
+extern "C" aio_status aio_pld_accept(const int* argmax, const int* draft, int* result, void* stream) {
+    if (!argmax || !draft || !result) return fail(AIO_ERR_INVALID_ARG, "argmax, draft and result must be non-NULL");
+    if ((reinterpret_cast<uintptr_t>(argmax) | reinterpret_cast<uintptr_t>(draft) | reinterpret_cast<uintptr_t>(result)) & 3u)
+        return fail(AIO_ERR_ALIGNMENT, "argmax, draft and result must be 4-byte aligned");
+    int dev = -1, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    AIO_CUDA(aio::launch_pld_accept(argmax, draft, result, static_cast<cudaStream_t>(stream)));
     return AIO_OK;
 }
