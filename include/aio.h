@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 4
+#define AIO_ABI_VERSION 5
 
 typedef enum {
     AIO_OK = 0,
@@ -316,6 +316,21 @@ aio_status aio_attention_check(void* workspace, int* device_error);
 aio_status aio_pld_draft(const int* tokens, int T, int N, int L, int* out, void* stream);
 aio_status aio_argmax_rows(const float* logits, int M, int V, int stride, int* out, void* stream);
 aio_status aio_pld_accept(const int* argmax, const int* draft, int* result, void* stream);
+
+/*
+ * The request-level routing decision (Sec. 3.2, Sec. 3.3) from the probe's single-token output.
+ * logits: the probe's fp32 logits over its vocabulary (device); category_tokens [n_categories]
+ * int32 (device): the token id of each category in the classification template; code_index: the
+ * category that is Code Generation.  On the device: the category is the argmax over the category
+ * logits (lowest index among ties); H is the softmax entropy over them in nats (the paper gives no
+ * base); the 1B model serves the request if it is Code Generation, L_ctx <= 2048 and H <= tau,
+ * the 7B model otherwise; PLD is on for every category but Code Generation.  decision [4] int32:
+ * category, model (1 or 7), PLD (1 on, 0 off), H as the bits of a float.  The paper's tau is 0.45.
+ * Errors: INVALID_ARG (NULL pointer, n_categories outside [1, 32], code_index outside them,
+ * negative L_ctx, tau negative or not finite), ALIGNMENT (a pointer not 4-byte aligned), CUDA.
+ */
+aio_status aio_route(const float* logits, const int* category_tokens, int n_categories, int code_index, int L_ctx,
+                     float tau, int* decision, void* stream);
 
 /*
  * Read-bandwidth probe: streams `bytes` from buf (device, 16-byte aligned, bytes a multiple of

@@ -42,7 +42,7 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
-AIO_ABI_VERSION = 4
+AIO_ABI_VERSION = 5
 AIO_X_GIVEN = 0
 AIO_X_RMSNORM = 1
 AIO_X_SWIGLU = 2
@@ -103,6 +103,7 @@ _SIGS = {
     "aio_pld_draft": (_int, [_vp, _int, _int, _int, _vp, _vp]),
     "aio_argmax_rows": (_int, [_vp, _int, _int, _int, _vp, _vp]),
     "aio_pld_accept": (_int, [_vp, _vp, _vp, _vp]),
+    "aio_route": (_int, [_vp, _vp, _int, _int, _int, ctypes.c_float, _vp, _vp]),
 }
 for _f, (_res, _args) in _SIGS.items():
     _fn = getattr(_lib, _f)
@@ -258,3 +259,8 @@ def aio_argmax_rows(logits: int, M: int, V: int, stride: int, out: int, stream: 
 
 def aio_pld_accept(argmax: int, draft: int, result: int, stream: int = 0):
     _check(_lib.aio_pld_accept(argmax, draft, result, stream), "aio_pld_accept")
+
+
+def aio_route(logits: int, category_tokens: int, n_categories: int, code_index: int, L_ctx: int, tau: float,
+              decision: int, stream: int = 0):
+    _check(_lib.aio_route(logits, category_tokens, n_categories, code_index, L_ctx, tau, decision, stream), "aio_route")

@@ -826,3 +826,22 @@ extern "C" aio_status aio_pld_accept(const int* argmax, const int* draft, int* r
     AIO_CUDA(aio::launch_pld_accept(argmax, draft, result, static_cast<cudaStream_t>(stream)));
     return AIO_OK;
 }
+
+extern "C" aio_status aio_route(const float* logits, const int* category_tokens, int n_categories, int code_index,
+                                int L_ctx, float tau, int* decision, void* stream) {
+    if (!logits || !category_tokens || !decision)
+        return fail(AIO_ERR_INVALID_ARG, "logits, category_tokens and decision must be non-NULL");
+    if (n_categories < 1 || n_categories > 32 || code_index < 0 || code_index >= n_categories || L_ctx < 0 ||
+        !(tau >= 0.0f) || !std::isfinite(tau))
+        return fail(AIO_ERR_INVALID_ARG, "need 1 <= n_categories <= 32, 0 <= code_index < n_categories, L_ctx >= 0, "
+                                         "finite tau >= 0");
+    if ((reinterpret_cast<uintptr_t>(logits) | reinterpret_cast<uintptr_t>(category_tokens) |
+         reinterpret_cast<uintptr_t>(decision)) & 3u)
+        return fail(AIO_ERR_ALIGNMENT, "logits, category_tokens and decision must be 4-byte aligned");
+    int dev = -1, sms = 0;
+    aio_status st = current_device(&dev, &sms);
+    if (st != AIO_OK) return st;
+    AIO_CUDA(aio::launch_route(logits, category_tokens, n_categories, code_index, L_ctx, tau, decision,
+                               static_cast<cudaStream_t>(stream)));
+    return AIO_OK;
+}

@@ -1,5 +1,6 @@
 // aio_pld.cu -- prompt-lookup decoding around the verification pass (Sec. 4.2: n-gram matching
-// window N = 6, look-ahead L = 2).  Three small kernels, all integer or comparison work:
+// window N = 6, look-ahead L = 2), and the routing decision.  Small kernels, mostly integer or
+// comparison work:
 //   * draft:  among positions i < T - 1, the one whose preceding tokens share the longest suffix
 //             (<= N) with the whole sequence, the most recent among equals; the draft is the up to
 //             L tokens after it.  One CTA: every thread scores positions i = tid, tid + 1024, ...
@@ -7,6 +8,9 @@
 //   * argmax: one CTA per row of logits; ties go to the lowest index, NaN counts as the maximum
 //             (the first NaN wins), as numpy's argmax does.
 //   * accept: greedy acceptance of the drafted tokens against the verification pass's argmax.
+//   * route:  the request-level decision of Sec. 3.2 and Sec. 3.3 from the probe's logits over the
+//             category tokens: category (argmax), softmax entropy in nats against tau, the model
+//             (1B only for confident Code Generation with L_ctx <= 2048) and the PLD switch.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -114,7 +118,47 @@ __global__ void aio_pld_accept_kernel(const int* __restrict__ argmax, const int*
     result[1] = argmax[a];
 }
 
+// One warp; lane c < n holds category c.
+__global__ void aio_route_kernel(const float* __restrict__ logits, const int* __restrict__ cat_tok, int n, int code,
+                                 int L_ctx, float tau, int* __restrict__ decision) {
+    const int lane = threadIdx.x;
+    const float l = lane < n ? logits[cat_tok[lane]] : -INFINITY;
+    float mx = l;
+    int arg = lane < n ? lane : 0x7FFFFFFF;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float om = __shfl_xor_sync(0xffffffffu, mx, o);
+        const int oa = __shfl_xor_sync(0xffffffffu, arg, o);
+        if (om > mx || (om == mx && oa < arg)) {
+            mx = om;
+            arg = oa;
+        }
+    }
+    const float e = lane < n ? expf(l - mx) : 0.0f;
+    float sum = e;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const float p = e / sum;
+    float t = p > 0.0f ? p * logf(p) : 0.0f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    const float H = -t;
+    if (lane == 0) {
+        const bool is_code = arg == code;
+        decision[0] = arg;
+        decision[1] = (is_code && L_ctx <= 2048 && H <= tau) ? 1 : 7;
+        decision[2] = is_code ? 0 : 1;
+        decision[3] = __float_as_int(H);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_route(const float* logits, const int* cat_tok, int n, int code, int L_ctx, float tau, int* decision,
+                         cudaStream_t s) {
+    aio_route_kernel<<<1, 32, 0, s>>>(logits, cat_tok, n, code, L_ctx, tau, decision);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_pld_draft(const int* tokens, int T, int N, int L, int* out, cudaStream_t s) {
     aio_pld_draft_kernel<<<1, kPldThreads, 0, s>>>(tokens, T, N, L, out);

@@ -12,5 +12,7 @@ constexpr int kPldMaxL = 7;    // longest look-ahead (the verification pass then
 cudaError_t launch_pld_draft(const int* tokens, int T, int N, int L, int* out, cudaStream_t s);
 cudaError_t launch_argmax(const float* logits, int M, int V, int stride, int* out, cudaStream_t s);
 cudaError_t launch_pld_accept(const int* argmax, const int* draft, int* result, cudaStream_t s);
+cudaError_t launch_route(const float* logits, const int* cat_tok, int n, int code, int L_ctx, float tau, int* decision,
+                         cudaStream_t s);
 
 }  // namespace aio

@@ -1,5 +1,6 @@
 """GPU parity of prompt-lookup decoding around the verification pass (aio_pld_draft, aio_argmax_rows,
-aio_pld_accept) against oracle/pld.py.  All three are integer or comparison work, so the bar is
+aio_pld_accept) against oracle/pld.py, and of the routing decision (aio_route) against
+oracle/route.py.  Drafting, argmax and acceptance are integer or comparison work, so the bar is
 bit-exact: the same draft length, matched n, position and tokens; the same argmax index; the same
 accepted count and next token.  Cases: sequences with many repeats (small vocabularies) and few
 (large), lengths from 1 to the paper's 32K context, every look-ahead up to 7, windows up to 32;
@@ -116,3 +117,32 @@ def test_argument_errors(aio):
         with pytest.raises(aio.AioError) as e:
             aio.aio_argmax_rows(*args, 0)
         assert e.value.status == status
+
+
+def test_route_matches_oracle(aio):
+    """aio_route against oracle/route.py: the category, the model and the PLD switch exactly (cases
+    within 1e-4 of the threshold are not compared: the fp32 sums there may round either way), the
+    entropy to 1e-5 relative."""
+    from oracle import route
+    rng = np.random.default_rng(3)
+    V = 32000
+    cases = 0
+    for trial in range(200):
+        n = int(rng.choice([2, 3, 5, 32]))
+        cat_tok = rng.choice(V, size=n, replace=False).astype(np.int32)
+        logits = rng.normal(scale=float(rng.choice([0.5, 2.0, 6.0])), size=V).astype(np.float32)
+        code = int(rng.integers(0, n))
+        L_ctx = int(rng.choice([0, 100, 2047, 2048, 2049, 32768]))
+        ld = torch.from_numpy(logits).cuda()
+        td = torch.from_numpy(cat_tok).cuda()
+        dec = torch.zeros(4, dtype=torch.int32, device="cuda")
+        aio.aio_route(ld.data_ptr(), td.data_ptr(), n, code, L_ctx, 0.45, dec.data_ptr(), 0)
+        c, m, pld_on, hbits = dec.cpu().tolist()
+        H = float(np.array([hbits], np.int32).view(np.float32)[0])
+        c_ref, H_ref, m_ref, pld_ref = route.route(logits[cat_tok], code, L_ctx)
+        assert c == c_ref and bool(pld_on) == pld_ref
+        assert abs(H - H_ref) <= 1e-5 * max(1.0, H_ref)
+        if abs(H_ref - 0.45) > 1e-4:
+            assert m == m_ref
+            cases += 1
+    assert cases > 150
