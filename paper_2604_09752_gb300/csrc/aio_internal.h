@@ -32,6 +32,9 @@
 #ifndef AIO_AHEAD_LIVE_I8
 #define AIO_AHEAD_LIVE_I8 2
 #endif
+#ifndef AIO_XBAR_ONLY
+#define AIO_XBAR_ONLY 1         // warps 1..7 learn of the grid barrier from the staged x's mbarrier (0: a shared flag)
+#endif
 #ifndef AIO_SLOT_KB_I8
 #define AIO_SLOT_KB_I8 AIO_SLOT_KB   // the same for int8 weights (4 KB tiles)
 #endif

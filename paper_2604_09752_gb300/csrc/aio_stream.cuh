@@ -1141,6 +1141,10 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 stage_x();
                 if (lane == 0) st_release_cta_shared(&cta_sync[1], static_cast<unsigned>(p));
                 if (polled && p > 1 && blockIdx.x == 0 && lane == 0) s.done[p - 2] = 0u;   // nobody polls it any more
+            } else if (AIO_XBAR_ONLY && stage && (!CH || P.xop == kXGiven)) {
+                // warp 0 stages x only after the grid counter is complete, so the staged x's
+                // barrier, waited on below, already orders this warp after the previous projection
+                ok = true;
             } else {
                 ok = poll_shared(&cta_sync[1], static_cast<unsigned>(p), s.wait_limit_ns, lane);
             }
