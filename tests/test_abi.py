@@ -89,3 +89,31 @@ def test_binding_fails_loudly_without_library(tmp_path):
     r = subprocess.run([sys.executable, "-c", "import paper_2604_09752_gb300.aio"], cwd=tmp_path,
                        capture_output=True, text=True)
     assert r.returncode != 0 and "libaio.so is missing" in r.stderr
+
+
+def test_new_entry_points_reject_bad_arguments_before_cuda(aio):
+    """The chained step, attention, PLD and routing entry points check their arguments on the host
+    and return before any CUDA call (these run without a GPU)."""
+    lib = aio.lib()
+    bad = aio.AIO_ERR_INVALID_ARG
+    assert lib.aio_decode_step_create_chained(None, None, None, 0, 1, 0) == bad
+    # attention: NULL pointers, then head_dim, M and L ranges, q_stride, alignment
+    assert lib.aio_attention_decode(None, 128, None, None, 1, 128, 16, 16, 1, None, None, 0, None) == bad
+    p = 1 << 20   # any non-NULL address: nothing is dereferenced before the checks below fail
+    assert lib.aio_attention_decode(p, 128, p, p, 1, 64, 16, 16, 1, p, p, 0, None) == aio.AIO_ERR_UNSUPPORTED
+    assert lib.aio_attention_decode(p, 128, p, p, 1, 128, 16, 16, 9, p, p, 0, None) == bad
+    assert lib.aio_attention_decode(p, 128, p, p, 1, 128, 16, 17, 1, p, p, 0, None) == bad
+    assert lib.aio_attention_decode(p, 64, p, p, 1, 128, 16, 16, 1, p, p, 0, None) == bad
+    assert lib.aio_attention_decode(p + 4, 128, p, p, 1, 128, 16, 16, 1, p, p, 0, None) == aio.AIO_ERR_ALIGNMENT
+    assert lib.aio_attention_workspace_bytes(9, None) == bad
+    # prompt lookup and routing
+    assert lib.aio_pld_draft(None, 10, 6, 2, None, None) == bad
+    assert lib.aio_pld_draft(p, 0, 6, 2, p, None) == bad
+    assert lib.aio_pld_draft(p, 10, 6, 8, p, None) == bad
+    assert lib.aio_pld_draft(p + 2, 10, 6, 2, p, None) == aio.AIO_ERR_ALIGNMENT
+    assert lib.aio_argmax_rows(p, 1, 10, 9, p, None) == bad
+    assert lib.aio_pld_accept(None, p, p, None) == bad
+    assert lib.aio_route(p, p, 0, 0, 10, ctypes.c_float(0.45), p, None) == bad
+    assert lib.aio_route(p, p, 3, 3, 10, ctypes.c_float(0.45), p, None) == bad
+    assert lib.aio_route(p, p, 3, 0, -1, ctypes.c_float(0.45), p, None) == bad
+    assert lib.aio_route(p, p, 3, 0, 10, ctypes.c_float(float("nan")), p, None) == bad
