@@ -4,7 +4,7 @@ Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline / reference leg
 module.  It shares no code with the CUDA path.  Plain Python over small integer lists.
 
 What it computes (Sec. 4.2 fixes the n-gram matching window N = 6 and the look-ahead L = 2; the
-paper prints no algorithm, so the steps below are the reading, also stated in the design doc):
+paper prints no algorithm, so the steps below are the reading):
 
   draft(tokens, N, L)
       For n = N, N-1, ..., 1: the last n tokens form the query.  Look for an earlier occurrence
