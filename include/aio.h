@@ -32,7 +32,10 @@
  *   - Devices: a handle or step belongs to the device that was current when it was
  *     created; using it while another device is current returns AIO_ERR_STATE.
  *   - Device-side waits are bounded.  A wait that expires sets an error word that
- *     aio_linear_check / aio_decode_step_check report as AIO_ERR_DEVICE_TIMEOUT.
+ *     aio_linear_check / aio_decode_step_check / aio_attention_check report as
+ *     AIO_ERR_DEVICE_TIMEOUT, with the code in *device_error: 1 a bulk-copy wait expired,
+ *     2 a wait for the previous projection expired, 3 a chained step's computed x did not fit
+ *     the staging area (refused on the host; the device check is a second guard).
  */
 #ifndef AIO_H
 #define AIO_H
