@@ -159,12 +159,21 @@ __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __g
             break;
         }
         {
+            // K and V rows are read from shared memory once for all tokens, and each step of the
+            // softmax runs for every token before the next, so the tokens' chains interleave.
             const int p0 = c * kAttnPos, np = min(kAttnPos, a.L - p0);
             const uint32_t kaddr = smem_addr(ring + cslot * kAttnSlot) + 8 * lane;
             const uint32_t vaddr = kaddr + kAttnUnitBytes;
-            uint2 kr[kAttnPos];
+            uint2 kr[kAttnPos], vr[kAttnPos];
 #pragma unroll
-            for (int j = 0; j < kAttnPos; ++j) kr[j] = j < np ? lds64(kaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+            for (int j = 0; j < kAttnPos; ++j) {
+                kr[j] = j < np ? lds64(kaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+                vr[j] = j < np ? lds64(vaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+            }
+            // lanes 2p and 2p + 1 hold position p's score (base-2 logits)
+            const int pos = (lane >> 1) & 15;
+            float sc[MT], bm[MT];
+            bool vis[MT];
 #pragma unroll
             for (int m = 0; m < MT; ++m) {
                 float part[kAttnPos];
@@ -174,36 +183,42 @@ __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __g
                     const float k2 = __uint_as_float(kr[j].y << 16), k3 = __uint_as_float(kr[j].y & 0xFFFF0000u);
                     part[j] = fmaf(q4[m].w, k3, fmaf(q4[m].z, k2, fmaf(q4[m].y, k1, q4[m].x * k0)));
                 }
-                // lanes 2p and 2p + 1 hold position p's score (base-2 logits)
-                const int pos = (lane >> 1) & 15;
-                float s = warp_sum16_transpose(part, lane);
-                const bool visible = pos < np && p0 + pos <= a.L - a.M + m;
-                s = visible ? s : -INFINITY;
-                float bm = s;
+                const float sm = warp_sum16_transpose(part, lane);
+                vis[m] = pos < np && p0 + pos <= a.L - a.M + m;
+                sc[m] = vis[m] ? sm : -INFINITY;
+                bm[m] = sc[m];
+            }
 #pragma unroll
-                for (int o = 2; o < 32; o <<= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
-                const float nm = fmaxf(mx[m], bm);
-                if (nm != -INFINITY) {
-                    const float alpha = exp2f(mx[m] - nm);   // 0 while mx is -inf
-                    const float p = visible ? exp2f(s - nm) : 0.0f;
-                    float psum = p;
+            for (int o = 2; o < 32; o <<= 1)
 #pragma unroll
-                    for (int o = 2; o < 32; o <<= 1) psum += __shfl_xor_sync(0xffffffffu, psum, o);
-                    ls[m] = ls[m] * alpha + psum;
-                    float4 ac = make_float4(acc[m].x * alpha, acc[m].y * alpha, acc[m].z * alpha, acc[m].w * alpha);
+                for (int m = 0; m < MT; ++m) bm[m] = fmaxf(bm[m], __shfl_xor_sync(0xffffffffu, bm[m], o));
+            float pr[MT], ps[MT];
 #pragma unroll
-                    for (int j = 0; j < kAttnPos; ++j) {
-                        const float pj = __shfl_sync(0xffffffffu, p, 2 * j);
-                        if (j < np) {
-                            const uint2 vr = lds64(vaddr + j * (kHeadDim * 2));
-                            ac.x = fmaf(pj, __uint_as_float(vr.x << 16), ac.x);
-                            ac.y = fmaf(pj, __uint_as_float(vr.x & 0xFFFF0000u), ac.y);
-                            ac.z = fmaf(pj, __uint_as_float(vr.y << 16), ac.z);
-                            ac.w = fmaf(pj, __uint_as_float(vr.y & 0xFFFF0000u), ac.w);
-                        }
-                    }
-                    acc[m] = ac;
-                    mx[m] = nm;
+            for (int m = 0; m < MT; ++m) {
+                const float nm = fmaxf(mx[m], bm[m]);
+                const bool live = nm != -INFINITY;   // some position seen so far is visible
+                const float alpha = live ? exp2f(mx[m] - nm) : 1.0f;   // 0 while mx is -inf
+                pr[m] = live && vis[m] ? exp2f(sc[m] - nm) : 0.0f;
+                ps[m] = pr[m];
+                ls[m] *= alpha;
+                acc[m] = make_float4(acc[m].x * alpha, acc[m].y * alpha, acc[m].z * alpha, acc[m].w * alpha);
+                if (live) mx[m] = nm;
+            }
+#pragma unroll
+            for (int o = 2; o < 32; o <<= 1)
+#pragma unroll
+                for (int m = 0; m < MT; ++m) ps[m] += __shfl_xor_sync(0xffffffffu, ps[m], o);
+#pragma unroll
+            for (int m = 0; m < MT; ++m) ls[m] += ps[m];
+#pragma unroll
+            for (int j = 0; j < kAttnPos; ++j) {
+                const float v0 = __uint_as_float(vr[j].x << 16), v1 = __uint_as_float(vr[j].x & 0xFFFF0000u);
+                const float v2 = __uint_as_float(vr[j].y << 16), v3 = __uint_as_float(vr[j].y & 0xFFFF0000u);
+#pragma unroll
+                for (int m = 0; m < MT; ++m) {
+                    const float pj = __shfl_sync(0xffffffffu, pr[m], 2 * j);   // 0 past np: V is zero there too
+                    acc[m] = make_float4(fmaf(pj, v0, acc[m].x), fmaf(pj, v1, acc[m].y), fmaf(pj, v2, acc[m].z),
+                                         fmaf(pj, v3, acc[m].w));
                 }
             }
         }
