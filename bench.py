@@ -218,6 +218,26 @@ def cpu_oracle_sample(wl, seed, frac, min_seconds=0.0):
     return dt, nbytes * passes, cores, passes
 
 
+def oracle_single_layer_ms():
+    """The oracle on the single 2048 x 2048 bf16 layer (M = 1), best of 5, with every host thread and
+    with one (a child process with OMP_NUM_THREADS=1): {"threads": n, "ms": t, "single_thread_ms": t1}."""
+    code = ("import sys, time; sys.path.insert(0, %r)\n"
+            "import oracle\n"
+            "from synth import workloads as swl\n"
+            "wl = swl.WORKLOADS['linear-2048']; p = wl.projs[0]\n"
+            "x = swl.gen_x(0, wl, p, 1).reshape(1, p.K); W = swl.gen_w_bf16(0, wl, p).reshape(p.N, p.K)\n"
+            "best = 1e9\n"
+            "for _ in range(5):\n"
+            "    t0 = time.perf_counter(); oracle.linear_bf16(x, W); best = min(best, time.perf_counter() - t0)\n"
+            "print(oracle.threads(), best * 1e3)\n") % ROOT
+    out = {}
+    for key, env in (("all", dict(os.environ)), ("one", dict(os.environ, OMP_NUM_THREADS="1"))):
+        r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=120)
+        threads, ms = r.stdout.split()
+        out[key] = (int(threads), float(ms))
+    return {"threads": out["all"][0], "ms": round(out["all"][1], 3), "single_thread_ms": round(out["one"][1], 3)}
+
+
 def run_reference(args, wl):
     world, rank, _ = dist_setup()
     if rank != 0:
@@ -247,6 +267,7 @@ def run_reference(args, wl):
         "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "gpu_launches": 0,
+        "oracle_linear_2048": oracle_single_layer_ms(),
     }
     print(json.dumps(line), flush=True)
     return 0
