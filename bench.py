@@ -274,6 +274,217 @@ def run_reference(args, wl):
 
 
 # ---------------------------------------------------------------------------------------------
+# ---------------------------------------------------------------------------------------------
+def time_calls(fn, stream, steps, warmup):
+    """Milliseconds per call of fn(stream handle): warmup untimed calls, then steps calls timed with
+    CUDA events on stream, with a device synchronize on both sides."""
+    import torch
+    sh = stream.cuda_stream
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            fn(sh)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(steps):
+            fn(sh)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def step_record(name, M, wtype, wbytes, ms, peak, launches, **extra):
+    """One sub-record of the configs block: a whole decode step of `name` at width M."""
+    gbs = wbytes / (ms / 1e3) / 1e9
+    r = {"workload": name, "M": M, "wtype": wtype, "weight_bytes_per_token": wbytes, "ms_per_step": round(ms, 4),
+         "GB/s": round(gbs, 2), "frac_of_measured_peak": round(gbs / peak, 4), "tokens_per_s": round(1000.0 / ms, 2),
+         "launches_per_step": launches}
+    if M > 1:
+        r["verified_tokens_per_s_upper_bound"] = round(1000.0 * M / ms, 2)
+    r.update(extra)
+    return r
+
+
+def bench_single_linear(args, peak):
+    """The single 2048 x 2048 bf16 layer at M = 1 (8.39 MB: it would sit in the 129 MB L2 if timed
+    alone), timed over 64 distinct seeded copies (537 MB, over 4x L2) so that every launch streams
+    from HBM.  Each copy is one standalone launch of the single-projection kernel (what
+    aio_linear_run enqueues), the 64 chained with programmatic dependent launch in one CUDA graph;
+    the time per layer is the graph's time / 64."""
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    from synth import workloads as swl
+    import torch
+    copies = 64
+    base = swl.WORKLOADS["linear-2048"].projs[0]
+    wl = swl.Workload("linear-2048-x64", 0, "bf16", 1, [swl.Proj(i, base.index, base.K, base.N) for i in range(copies)],
+                      "64 distinct copies of the single 2048 x 2048 layer")
+    dw = DeviceWorkload(wl, seed=args.seed, max_M=1)
+    dw.fill_x(1)
+    step = dw.step_handle(1, aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL)
+    stream = torch.cuda.Stream()
+    ms = time_calls(lambda sh: aio.aio_decode_step(step, sh), stream, args.steps, args.warmup)
+    assert aio.aio_decode_step_check(step) == 0
+    dw.close()
+    layer = base.N * base.K * 2
+    per = ms / copies
+    gbs = layer / (per / 1e3) / 1e9
+    return {"workload": "linear-2048", "baseline_config": 1, "M": 1, "wtype": "bf16", "weight_bytes_per_layer": layer,
+            "ms_per_layer": round(per, 5), "GB/s": round(gbs, 2), "frac_of_measured_peak": round(gbs / peak, 4),
+            "copies": copies, "rotating_weight_bytes": copies * layer, "launches_per_layer": 1,
+            "l2": "64 distinct copies, 537 MB, over 4x the 129 MB L2"}
+
+
+def bench_steps(args, peak, wl, widths, name_of, **extra):
+    """Whole decode steps of one weight set at each width M (one persistent launch per step)."""
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    import torch
+    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
+    dw = DeviceWorkload(wl, seed=args.seed, max_M=max(widths))
+    wbytes = dw.weight_bytes()
+    stream = torch.cuda.Stream()
+    out = {}
+    for M in widths:
+        dw.fill_x(M)
+        step = dw.step_handle(M, flags)
+        ms = time_calls(lambda sh: aio.aio_decode_step(step, sh), stream, args.steps, args.warmup)
+        assert aio.aio_decode_step_check(step) == 0
+        out[name_of(M)] = step_record(name_of(M), M, wl.wtype, wbytes, ms, peak, aio.aio_decode_step_kernels(step),
+                                      **extra)
+    dw.close()
+    return out
+
+
+def bench_chain(args, peak):
+    """The chained 7B-class decoder step (every x computed on the device from earlier outputs:
+    RMSNorm with residual adds, V of QKV, SwiGLU), M = 1, one persistent launch per step."""
+    from paper_2604_09752_gb300 import aio
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    from synth import workloads as swl
+    import torch
+    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
+    out = {}
+    for name in ("7b-bf16", "7b-int8"):
+        wl = swl.WORKLOADS[name]
+        dw = DeviceWorkload(wl, seed=args.seed, max_M=1, chained=True)
+        dw.fill_chain(1)
+        step = dw.step_handle(1, flags)
+        stream = torch.cuda.Stream()
+        ms = time_calls(lambda sh: aio.aio_decode_step(step, sh), stream, args.steps, args.warmup)
+        assert aio.aio_decode_step_check(step) == 0
+        key = f"7b-chain-{wl.wtype}"
+        out[key] = step_record(key, 1, wl.wtype, dw.weight_bytes(), ms, peak, aio.aio_decode_step_kernels(step))
+        dw.close()
+    return out
+
+
+def bench_attention(args, peak):
+    """Decode attention over KV caches of the 7B-class shapes (32 heads x 128) at the paper's 2K and
+    32K contexts, M = 1 and 3 (PLD look-ahead L = 2): one call per layer, over enough distinct layer
+    caches (seeded bf16 N(0, 1)) that a step streams more than 1 GB, well above L2; a step's calls
+    are captured in one CUDA graph.  Metric: KV bytes per step / time."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    n_heads, d = 32, 128
+    gen = torch.Generator(device="cuda").manual_seed(args.seed)
+    stream = torch.cuda.Stream()
+    out = {}
+    for L, layers in ((2048, 32), (32768, 4)):
+        caches = [(torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16),
+                   torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16)) for _ in range(layers)]
+        for M in (1, 3):
+            q = torch.randn(M, n_heads * d, device="cuda", generator=gen)
+            o = torch.empty(M, n_heads * d, device="cuda")
+            wsb = aio.aio_attention_workspace_bytes(M)
+            ws = torch.zeros(wsb, dtype=torch.uint8, device="cuda")
+
+            def one_step(sh):
+                for kc, vc in caches:
+                    aio.aio_attention_decode(q.data_ptr(), n_heads * d, kc.data_ptr(), vc.data_ptr(), n_heads, d, L, L, M,
+                                             o.data_ptr(), ws.data_ptr(), wsb, sh)
+            torch.cuda.synchronize()
+            one_step(stream.cuda_stream)
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()            # one replay per step: no host gaps between layers
+            with torch.cuda.graph(graph, stream=stream):
+                one_step(stream.cuda_stream)
+            torch.cuda.synchronize()
+            ms = time_calls(lambda sh: graph.replay(), stream, args.steps, args.warmup)
+            assert aio.aio_attention_check(ws.data_ptr()) == 0
+            kv_bytes = layers * 2 * n_heads * L * d * 2
+            gbs = kv_bytes / (ms / 1e3) / 1e9
+            key = f"7b-attention-L{L}-M{M}"
+            out[key] = {"workload": key, "L": L, "M": M, "layers": layers, "ms_per_step": round(ms, 4),
+                        "ms_per_layer": round(ms / layers, 5), "kv_bytes_per_step": kv_bytes, "GB/s": round(gbs, 2),
+                        "frac_of_measured_peak": round(gbs / peak, 4), "launches_per_layer": 2}
+        del caches
+        torch.cuda.empty_cache()
+    return out
+
+
+def bench_pld_ops(args):
+    """Latency of the work around a PLD verification pass (Sec. 4.2, N = 6, L = 2): drafting over a
+    2K and a 32K token history, the argmax of 3 rows of 32000 logits, and the acceptance check;
+    each captured in a CUDA graph and replayed, so the figure is device time per call."""
+    import torch
+    from paper_2604_09752_gb300 import aio
+    gen = torch.Generator(device="cuda").manual_seed(args.seed)
+    stream = torch.cuda.Stream()
+    res = {}
+    for name, T in (("draft_2k", 2048), ("draft_32k", 32768)):
+        toks = torch.randint(0, 32000, (T,), dtype=torch.int32, device="cuda", generator=gen)
+        out = torch.zeros(5, dtype=torch.int32, device="cuda")
+        res[name] = (lambda t=toks, o=out, n=T: aio.aio_pld_draft(t.data_ptr(), n, 6, 2, o.data_ptr(), stream.cuda_stream))
+    logits = torch.randn(3, 32000, device="cuda", generator=gen)
+    am = torch.zeros(3, dtype=torch.int32, device="cuda")
+    res["argmax_3x32000"] = lambda: aio.aio_argmax_rows(logits.data_ptr(), 3, 32000, 32000, am.data_ptr(), stream.cuda_stream)
+    dbuf = torch.tensor([2, 2, 0, 1, 2], dtype=torch.int32, device="cuda")
+    acc = torch.zeros(2, dtype=torch.int32, device="cuda")
+    res["accept"] = lambda: aio.aio_pld_accept(am.data_ptr(), dbuf.data_ptr(), acc.data_ptr(), stream.cuda_stream)
+    line = {"unit": "us per call"}
+    for name, fn in res.items():
+        reps = 50
+        fn()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        torch.cuda.synchronize()
+        line[name] = round(time_calls(lambda sh: g.replay(), stream, 3, 1) * 1e3 / reps, 2)
+    return line
+
+
+def configs_block(args, peak, local, main_rec):
+    """Every BASELINE config in one object (configs 1 to 5), then the later rows of the path (chained
+    step, decode attention, PLD drafting and acceptance), with the clocks seen meanwhile."""
+    from synth import workloads as swl
+    clocks = ClockSampler(local)
+    t0 = time.time()
+    out = {"linear-2048": bench_single_linear(args, peak)}
+    out.update(bench_steps(args, peak, swl.WORKLOADS["1b-bf16"], (1,), lambda M: "1b-bf16", baseline_config=2))
+    out["7b-bf16"] = dict(main_rec, baseline_config=3, measured_in="the main line above")
+    for wt in ("bf16", "int8"):
+        out.update(bench_steps(args, peak, swl.pld_workload(8, wt), swl.PLD_WIDTHS,
+                               lambda M, wt=wt: f"7b-pld-{wt}-M{M}", baseline_config=5))
+    m1 = out["7b-pld-int8-M1"]
+    out["7b-int8"] = dict(m1, workload="7b-int8", baseline_config=4,
+                          measured_in="the int8 weight set of the PLD sweep at M = 1 (the same kernel and launch)")
+    if args.configs == "all":
+        nxt = {}
+        nxt.update(bench_chain(args, peak))
+        nxt.update(bench_attention(args, peak))
+        nxt["pld_ops"] = bench_pld_ops(args)
+        out["next_rows"] = nxt
+    out["clocks"] = clocks.stop(t0, time.time())
+    out["steps"], out["warmup"] = args.steps, args.warmup
+    return out
+
+
+# ---------------------------------------------------------------------------------------------
 def run_ours(args, wl):
     import torch
     world, rank, local = dist_setup()
@@ -326,65 +537,49 @@ def run_ours(args, wl):
     value, ms_max = replica_throughput(pg, wbytes, ms)
     assert aio.aio_decode_step_check(step) == 0
 
-    # ---- end to end: pinned host x -> device, step, device y -> pinned host, every step
+    # ---- end to end through the public API: aio_decode_step_host copies the step's x from pinned
+    # host memory, runs the step and copies its y back to pinned host memory, every step
     y_host = torch.empty(dw.y_arena.numel(), dtype=torch.uint8, pin_memory=True)
-    for _ in range(3):
-        with torch.cuda.stream(stream):
-            dw.x_arena.copy_(x_host, non_blocking=True)
-            aio.aio_decode_step(step, sh)
-            y_host.copy_(dw.y_arena, non_blocking=True)
-    torch.cuda.synchronize()
+    xb, yb = x_host.numel(), y_host.numel()
+
+    def e2e_step(s):
+        aio.aio_decode_step_host(step, x_host.data_ptr(), dw.x_arena.data_ptr(), xb, dw.y_arena.data_ptr(),
+                                 y_host.data_ptr(), yb, s)
     e_steps = max(10, args.steps // 4)
     barrier(pg)
-    torch.cuda.synchronize()
-    ev0.record(stream)
-    with torch.cuda.stream(stream):
-        for _ in range(e_steps):
-            dw.x_arena.copy_(x_host, non_blocking=True)
-            aio.aio_decode_step(step, sh)
-            y_host.copy_(dw.y_arena, non_blocking=True)
-    ev1.record(stream)
-    torch.cuda.synchronize()
+    e_ms_rank = time_calls(e2e_step, stream, e_steps, 3)
     barrier(pg)
-    e2e_gbs, e_ms = replica_throughput(pg, wbytes, ev0.elapsed_time(ev1) / e_steps)
+    e2e_gbs, e_ms = replica_throughput(pg, wbytes, e_ms_rank)
+    assert torch.equal(y_host, dw.y_arena.cpu()), "host copy of y differs from the device's"
 
     # ---- largest projection alone (standalone kernel, same stream)
     big = max(range(len(dw.bufs)), key=lambda i: dw.bufs[i].proj.N * dw.bufs[i].proj.K)
     bp = dw.bufs[big].proj
-    with torch.cuda.stream(stream):
-        for _ in range(5):
-            dw.run_proj(big, M, sh)
-    reps = 50
-    ev0.record(stream)
-    with torch.cuda.stream(stream):
-        for _ in range(reps):
-            dw.run_proj(big, M, sh)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    big_ms = ev0.elapsed_time(ev1) / reps
+    big_ms = time_calls(lambda s: dw.run_proj(big, M, s), stream, 50, 5)
     esize = 1 if dw.i8 else 2
     big_bytes = bp.N * bp.K * esize + (2 * bp.N if dw.i8 else 0)
 
     # ---- read ceiling of the same bulk-copy ring (4 GiB, well above L2)
     pbuf = torch.empty(4 << 30, dtype=torch.uint8, device="cuda")
     pout = torch.zeros(1, dtype=torch.int32, device="cuda")
-    for _ in range(3):
-        aio.aio_probe_read(pbuf.data_ptr(), pbuf.numel(), pout.data_ptr(), sh)
-    ev0.record(stream)
-    for _ in range(10):
-        aio.aio_probe_read(pbuf.data_ptr(), pbuf.numel(), pout.data_ptr(), sh)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    probe_gbs = pbuf.numel() * 10 / (ev0.elapsed_time(ev1) / 1e3) / 1e9
+    probe_ms = time_calls(lambda s: aio.aio_probe_read(pbuf.data_ptr(), pbuf.numel(), pout.data_ptr(), s), stream, 10, 3)
+    probe_gbs = pbuf.numel() / (probe_ms / 1e3) / 1e9
     del pbuf
 
     peak, peak_src = measured_peak()
     gbs_rank = wbytes / (ms / 1e3) / 1e9
     tokens = world * 1000.0 / ms_max
     traffic, traffic_note = committed_traffic(wl.name, n_kernels)
+    dw.close()
+    del dw
+    torch.cuda.empty_cache()
 
     line = None
     if rank == 0:
+        main_rec = step_record(wl.name, M, wl.wtype, wbytes, ms, peak, n_kernels)
+        configs = None
+        if world == 1 and args.configs != "none":
+            configs = configs_block(args, peak, local, main_rec)
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             dt, nbytes, cores, passes = cpu_oracle_sample(wl, args.seed, args.cpu_frac, args.cpu_seconds)
@@ -402,12 +597,12 @@ def run_ours(args, wl):
             "higher_is_better": True,
             "scaling": "weak",
             "vs_baseline": None,
-            "dtype": "int8" if dw.i8 else "bf16",
+            "dtype": "int8" if wl.wtype == "int8" else "bf16",
             "data": "synthetic",
             "config": {
                 "workload": wl.name,
                 "description": wl.description,
-                "M": M, "wtype": wl.wtype, "projections": len(dw.bufs),
+                "M": M, "wtype": wl.wtype, "projections": len(wl.projs),
                 "weight_bytes_per_token": wbytes,
                 "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                 "l2": "inputs larger than L2 (every step streams all weights, >= 2.39 GB)",
@@ -419,7 +614,7 @@ def run_ours(args, wl):
             "pct_of_nominal_8tbs": round(100 * gbs_rank / NOMINAL_HBM_GBS, 2),
             "roofline": {
                 "bound": "hbm",
-                "kernel": f"aio_stream_kernel<M={M}, {'int8' if dw.i8 else 'bf16'}>",
+                "kernel": f"aio_stream_kernel<M={M}, {wl.wtype}>",
                 "achieved": round(gbs_rank, 2),
                 "peak": peak,
                 "unit": "GB/s",
@@ -435,196 +630,23 @@ def run_ours(args, wl):
                              "GB/s": round(big_bytes / (big_ms / 1e3) / 1e9, 2)},
             "probe_read_gbs": round(probe_gbs, 1),
             "e2e": {"value": round(e2e_gbs, 2), "unit": "GB/s", "ms_per_step": round(e_ms, 4),
-                    "h2d_bytes_per_step": int(dw.x_arena.numel()), "d2h_bytes_per_step": int(dw.y_arena.numel()),
-                    "path": "pinned host x -> aio_decode_step -> pinned host y, same stream"},
+                    "h2d_bytes_per_step": int(xb), "d2h_bytes_per_step": int(yb),
+                    "path": "aio_decode_step_host: pinned host x -> device, the step, device y -> pinned host, "
+                            "one stream"},
             "gpu_launches": args.steps * n_kernels,
             "clocks": clk,
             "setup_s": round(setup_s, 1),
             "cpu_baseline": cpu,
+            "configs": configs,
             # The paper's own decode rates on Ascend 910B, FP16 at 2K context (Tab. 3, Tab. 4): context only.
             "paper_context": {"hardware": "Ascend 910B", "tokens_per_s_1b": 21.58, "tokens_per_s_7b": 17.18,
                               "tokens_per_s_a_io_scenario_a": 19.80},
         }
         print(json.dumps(line), flush=True)
-    dw.close()
-    if args.pld_sweep and rank == 0:
-        pld_sweep(args, peak)
-        pld_ops_line(args)
-    if args.chain and rank == 0:
-        chain_lines(args, peak)
-    if args.attention and rank == 0:
-        attention_lines(args, peak)
     if pg is not None:
+        pg.barrier()
         pg.destroy_process_group()
     return 0
-
-
-def pld_sweep(args, peak):
-    """Prompt-lookup verification widths (Sec. 4.2): the 7B-class step at M = 1, 2, 4, 8 for bf16 and
-    int8 weights, one weight set per type, one JSON line per (type, M) after the main line."""
-    import torch
-    from paper_2604_09752_gb300 import aio
-    from paper_2604_09752_gb300.workload import DeviceWorkload
-    from synth import workloads as swl
-    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
-    for wt in ("bf16", "int8"):
-        wl = swl.pld_workload(8, wt)
-        dw = DeviceWorkload(wl, seed=args.seed, max_M=8)
-        wbytes = dw.weight_bytes()
-        stream = torch.cuda.Stream()
-        for M in swl.PLD_WIDTHS:
-            dw.fill_x(M)
-            step = dw.step_handle(M, flags)
-            with torch.cuda.stream(stream):
-                for _ in range(args.warmup):
-                    aio.aio_decode_step(step, stream.cuda_stream)
-            torch.cuda.synchronize()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for _ in range(args.steps):
-                aio.aio_decode_step(step, stream.cuda_stream)
-            e1.record(stream)
-            torch.cuda.synchronize()
-            assert aio.aio_decode_step_check(step) == 0
-            ms = e0.elapsed_time(e1) / args.steps
-            gbs = wbytes / (ms / 1e3) / 1e9
-            print(json.dumps({"sweep": "pld", "workload": f"7b-pld-{wt}-M{M}", "M": M, "wtype": wt,
-                              "ms_per_step": round(ms, 4), "value": round(gbs, 2), "unit": "GB/s",
-                              "frac_of_measured_peak": round(gbs / peak, 4),
-                              "tokens_per_s": round(1000.0 / ms, 2),
-                              "verified_tokens_per_s_upper_bound": round(1000.0 * M / ms, 2),
-                              "steps": args.steps, "warmup": args.warmup}), flush=True)
-        dw.close()
-
-
-def pld_ops_line(args):
-    """Latency of the work around a PLD verification pass (Sec. 4.2, N = 6, L = 2): drafting over a
-    2K and a 32K token history, the argmax of 3 rows of 32000 logits, and the acceptance check;
-    each captured in a CUDA graph and replayed, so the figure is device time per call."""
-    import torch
-    from paper_2604_09752_gb300 import aio
-    gen = torch.Generator(device="cuda").manual_seed(args.seed)
-    stream = torch.cuda.Stream()
-    res = {}
-    for name, T in (("draft_2k", 2048), ("draft_32k", 32768)):
-        toks = torch.randint(0, 32000, (T,), dtype=torch.int32, device="cuda", generator=gen)
-        out = torch.zeros(5, dtype=torch.int32, device="cuda")
-        res[name] = (lambda t=toks, o=out, n=T: aio.aio_pld_draft(t.data_ptr(), n, 6, 2, o.data_ptr(), stream.cuda_stream))
-    logits = torch.randn(3, 32000, device="cuda", generator=gen)
-    am = torch.zeros(3, dtype=torch.int32, device="cuda")
-    res["argmax_3x32000"] = lambda: aio.aio_argmax_rows(logits.data_ptr(), 3, 32000, 32000, am.data_ptr(), stream.cuda_stream)
-    dbuf = torch.tensor([2, 2, 0, 1, 2], dtype=torch.int32, device="cuda")
-    acc = torch.zeros(2, dtype=torch.int32, device="cuda")
-    res["accept"] = lambda: aio.aio_pld_accept(am.data_ptr(), dbuf.data_ptr(), acc.data_ptr(), stream.cuda_stream)
-    line = {"sweep": "pld_ops", "unit": "us per call"}
-    for name, fn in res.items():
-        reps = 50
-        fn()
-        torch.cuda.synchronize()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            for _ in range(reps):
-                fn()
-        g.replay()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        with torch.cuda.stream(stream):
-            g.replay()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        line[name] = round(e0.elapsed_time(e1) * 1e3 / reps, 2)
-    print(json.dumps(line), flush=True)
-
-
-def chain_lines(args, peak):
-    """The chained 7B-class decoder step (every x computed on the device from earlier outputs:
-    RMSNorm with residual adds, V of QKV, SwiGLU), M = 1, one persistent launch per step; one
-    JSON line per weight type after the main line."""
-    import torch
-    from paper_2604_09752_gb300 import aio
-    from paper_2604_09752_gb300.workload import DeviceWorkload
-    from synth import workloads as swl
-    flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
-    for name in ("7b-bf16", "7b-int8"):
-        dw = DeviceWorkload(swl.WORKLOADS[name], seed=args.seed, max_M=1, chained=True)
-        dw.fill_chain(1)
-        wbytes = dw.weight_bytes()
-        step = dw.step_handle(1, flags)
-        stream = torch.cuda.Stream()
-        with torch.cuda.stream(stream):
-            for _ in range(args.warmup):
-                aio.aio_decode_step(step, stream.cuda_stream)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(args.steps):
-            aio.aio_decode_step(step, stream.cuda_stream)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        assert aio.aio_decode_step_check(step) == 0
-        ms = e0.elapsed_time(e1) / args.steps
-        gbs = wbytes / (ms / 1e3) / 1e9
-        print(json.dumps({"sweep": "chain", "workload": f"7b-chain-{swl.WORKLOADS[name].wtype}", "M": 1,
-                          "ms_per_step": round(ms, 4), "value": round(gbs, 2), "unit": "GB/s",
-                          "frac_of_measured_peak": round(gbs / peak, 4), "tokens_per_s": round(1000.0 / ms, 2),
-                          "launches_per_step": aio.aio_decode_step_kernels(step), "steps": args.steps,
-                          "warmup": args.warmup}), flush=True)
-        dw.close()
-
-
-def attention_lines(args, peak):
-    """Decode attention over KV caches of the 7B-class shapes (32 heads x 128) at the paper's 2K and
-    32K contexts, M = 1 and 3 (PLD look-ahead L = 2): one call per layer, over enough distinct layer
-    caches (seeded bf16 N(0, 1)) that a step streams more than 1 GB, well above L2; a step's calls
-    are captured in one CUDA graph.  One JSON line per (context, M): KV bytes per step / time."""
-    import torch
-    from paper_2604_09752_gb300 import aio
-    n_heads, d = 32, 128
-    gen = torch.Generator(device="cuda").manual_seed(args.seed)
-    stream = torch.cuda.Stream()
-    for L, layers in ((2048, 32), (32768, 4)):
-        caches = [(torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16),
-                   torch.randn(n_heads * L * d, device="cuda", generator=gen).to(torch.bfloat16)) for _ in range(layers)]
-        for M in (1, 3):
-            q = torch.randn(M, n_heads * d, device="cuda", generator=gen)
-            out = torch.empty(M, n_heads * d, device="cuda")
-            wsb = aio.aio_attention_workspace_bytes(M)
-            ws = torch.zeros(wsb, dtype=torch.uint8, device="cuda")
-
-            def step():
-                for kc, vc in caches:
-                    aio.aio_attention_decode(q.data_ptr(), n_heads * d, kc.data_ptr(), vc.data_ptr(), n_heads, d, L, L, M,
-                                             out.data_ptr(), ws.data_ptr(), wsb, stream.cuda_stream)
-            torch.cuda.synchronize()
-            for _ in range(args.warmup):
-                step()
-            torch.cuda.synchronize()
-            graph = torch.cuda.CUDAGraph()            # one replay per step: no host gaps between layers
-            with torch.cuda.graph(graph, stream=stream):
-                step()
-            torch.cuda.synchronize()
-            for _ in range(args.warmup):
-                graph.replay()
-            torch.cuda.synchronize()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            with torch.cuda.stream(stream):
-                for _ in range(args.steps):
-                    graph.replay()
-            e1.record(stream)
-            torch.cuda.synchronize()
-            assert aio.aio_attention_check(ws.data_ptr()) == 0
-            ms = e0.elapsed_time(e1) / args.steps
-            kv_bytes = layers * 2 * n_heads * L * d * 2
-            gbs = kv_bytes / (ms / 1e3) / 1e9
-            print(json.dumps({"sweep": "attention", "workload": f"7b-attention-L{L}-M{M}", "L": L, "M": M,
-                              "layers": layers, "ms_per_step": round(ms, 4), "ms_per_layer": round(ms / layers, 5),
-                              "kv_bytes_per_step": kv_bytes, "value": round(gbs, 2), "unit": "GB/s",
-                              "frac_of_measured_peak": round(gbs / peak, 4), "launches_per_layer": 2,
-                              "steps": args.steps, "warmup": args.warmup}), flush=True)
-        del caches
-        torch.cuda.empty_cache()
 
 
 def main():
@@ -639,12 +661,9 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="repeat oracle passes over the row sample for at least this long")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--pld-sweep", action="store_true",
-                    help="after the main line, one line per PLD width M in {1,2,4,8} for bf16 and int8 7B steps")
-    ap.add_argument("--chain", action="store_true",
-                    help="after the main line, the chained 7B decoder step (x computed on the device), bf16 and int8")
-    ap.add_argument("--attention", action="store_true",
-                    help="after the main line, decode attention over 7B-shaped KV caches at 2K and 32K contexts")
+    ap.add_argument("--configs", choices=["all", "baseline", "none"], default="all",
+                    help="the configs block (N = 1 only): every BASELINE config (baseline), plus the chained step, "
+                         "decode attention and PLD drafting (all), or nothing (none)")
     ap.add_argument("--step-mode", choices=["persistent", "chain"], default="persistent",
                     help="one cooperative launch per step (default) or one launch per projection")
     args = ap.parse_args()

@@ -47,7 +47,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 5
+#define AIO_ABI_VERSION 6
 
 typedef enum {
     AIO_OK = 0,
@@ -155,7 +155,9 @@ const char* aio_last_error(void);
  */
 aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int max_M, unsigned flags);
 
-/* Bytes of the packed weight buffer (N*K*elem_size) and of the scale buffer (2*N for int8, else 0). */
+/* Bytes of the packed weight buffer (N*K*elem_size) and of the scale buffer (2*N for int8, else 0):
+ * the bytes every decode step streams for this layer (Sec. 3.1), half of them for the int8 codes
+ * of storage-only quantization (Sec. 2.4) plus their per-channel scales. */
 aio_status aio_linear_packed_bytes(aio_linear_t h, size_t* w_bytes, size_t* scale_bytes);
 
 /* Launch geometry of aio_linear_run: CTAs, threads per CTA, dynamic shared memory bytes,
@@ -163,6 +165,8 @@ aio_status aio_linear_packed_bytes(aio_linear_t h, size_t* w_bytes, size_t* scal
 aio_status aio_linear_launch_info(aio_linear_t h, int* grid, int* block, size_t* smem_bytes, long long* tiles);
 
 /*
+ * Store a layer's weights for streaming (Sec. 2.1: every decode step reads them all from HBM; Sec.
+ * 2.4: int8 weights are stored as codes plus scales and dequantized only inside the kernel).
  * Pack row-major W [N, K] (bf16 or int8, device) into the tiled layout above (device,
  * aio_linear_packed_bytes bytes, must not overlap W).  For int8, scales [N] bf16 are copied
  * to scales_packed (both device, or both NULL for bf16).  All pointers 16-byte aligned.
@@ -200,12 +204,17 @@ aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, co
  *   K, N          as for aio_linear_create
  *   wt            AIO_W_BF16 or AIO_W_INT8_PERCHANNEL
  *   flags         AIO_FLAG_ROWMAJOR and / or AIO_FLAG_NO_PDL
- *   device_error  device int, 4-byte aligned, owned by the caller: set non-zero if a bounded
- *                 device-side wait expired (y is then incomplete); the library never clears it
+ *   device_error  device int, 4-byte aligned, owned by the caller.  It must hold 0 when the call
+ *                 runs on the stream.  The kernel sets it non-zero if a bounded device-side wait
+ *                 expired (y is then incomplete).  The library never clears it, so an error stays
+ *                 visible to the caller across later calls; but while it is non-zero, later calls
+ *                 that share the word give up at their first wait for another warp's partial sums
+ *                 and leave y incomplete.  Clear it (e.g. cudaMemsetAsync) before reusing it.
  * Scratch: the cross-warp partial sums live in one static device array of
- * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs 512 M S
- * bytes of it (S = the device's SM count), rounded up to 256: on a 152-SM GB300 every M <= 8 fits
- * (622592 bytes at M = 8).  A call that needs more returns AIO_ERR_INVALID_ARG and launches nothing.
+ * AIO_NOALLOC_SCRATCH_BYTES per device, part of the loaded library image.  A call needs
+ * 16 * 4 * M * Z bytes of it, rounded up to 256, where Z = the device's SM count times the warps per
+ * CTA (8 in the default build): on a 152-SM GB300 every M <= 8 fits (622592 bytes at M = 8).  A call
+ * that needs more returns AIO_ERR_INVALID_ARG and launches nothing.
  * Each call enqueues a cudaMemsetAsync that empties the partial-sum slots it uses (all bytes 0xFF),
  * then the kernel.
  * Every call on a device shares that scratch: calls that overlap in time race and give wrong
@@ -226,7 +235,8 @@ aio_status aio_linear_check(aio_linear_t h, int* device_error);
 /* Empty the handle's partial-sum slots and clear its error word (needed only after a device error). */
 aio_status aio_linear_reset(aio_linear_t h);
 
-/* Free the handle and its workspace (synchronises the device). NULL is accepted. */
+/* Free the handle of one linear layer (Sec. 2.1) and its workspace (synchronises the device).
+ * NULL is accepted. */
 aio_status aio_linear_destroy(aio_linear_t h);
 
 /*
@@ -256,6 +266,18 @@ aio_status aio_decode_step_create_chained(aio_step_t* out, const aio_proj* projs
 /* Enqueue one decode step on stream (one graph launch with AIO_STEP_GRAPH). */
 aio_status aio_decode_step(aio_step_t step, void* stream);
 
+/*
+ * One decode step from host memory (Sec. 3.1: one generated token): copy x_bytes from x_host to
+ * x_dev, run the step, copy y_bytes from y_dev to y_host, all in order on stream.  x_dev and y_dev
+ * are device buffers the step reads and writes (e.g. one arena holding every projection's x, and
+ * one holding every y); x_host and y_host are host buffers, page-locked for the copies to be
+ * asynchronous.  A size of 0 skips that copy.  Returns without synchronising: y_host is valid once
+ * the stream has executed the work.  Errors: INVALID_ARG (a copy of non-zero size with a NULL
+ * pointer), STATE, CUDA.
+ */
+aio_status aio_decode_step_host(aio_step_t step, const void* x_host, void* x_dev, size_t x_bytes, const void* y_dev,
+                                void* y_host, size_t y_bytes, void* stream);
+
 /* Number of kernels one aio_decode_step launches (1 in persistent mode, else one per projection). */
 aio_status aio_decode_step_kernels(aio_step_t step, int* n_kernels);
 
@@ -265,7 +287,8 @@ aio_status aio_decode_step_reset(aio_step_t step);
 /* Synchronise the device, then report the step's device error word (see aio_linear_check). */
 aio_status aio_decode_step_check(aio_step_t step, int* device_error);
 
-/* Free the step, its graph and its workspace (synchronises the device). NULL is accepted. */
+/* Free a decode step (Sec. 3.1), its graph and its workspace (synchronises the device). NULL is
+ * accepted. */
 aio_status aio_decode_step_destroy(aio_step_t step);
 
 /*

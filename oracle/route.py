@@ -12,8 +12,9 @@ The probe model emits one categorical token; from its logits over the category t
     model otherwise (General QA / Math, long contexts, or H > tau);
   * PLD: on for every request that is not Code Generation (they all go to the 7B model), off for
     Code Generation whichever model serves it.
-Where the entropy decides the model, it is computed in float32, the precision of the CUDA path,
-with the same formula: p_c = exp(l_c - max) / sum, H = -sum p_c ln p_c over p_c > 0.
+The entropy is the plain definition evaluated in double: p_c = exp(l_c) / sum_j exp(l_j) (shifted
+by the largest logit, which leaves p unchanged and keeps exp finite), H = -sum_c p_c ln p_c over the
+p_c > 0 (0 ln 0 = 0).  The threshold compares H <= tau in double.
 
 Parity status: pinned by tests/test_oracle_route_pins.py (closed forms of the entropy and the
 decision table of Sec. 3.3).
@@ -28,19 +29,19 @@ MODEL_1B, MODEL_7B = 1, 7
 
 
 def entropy(cat_logits) -> float:
-    """Softmax entropy in nats, evaluated in float32."""
-    l = np.asarray(cat_logits, dtype=np.float32)
-    e = np.exp(l - l.max(), dtype=np.float32)
-    p = e / e.sum(dtype=np.float32)
+    """Softmax entropy in nats, evaluated in double."""
+    l = np.asarray(cat_logits, dtype=np.float64)
+    e = np.exp(l - l.max())
+    p = e / e.sum()
     nz = p[p > 0]
-    return float(-np.sum(nz * np.log(nz), dtype=np.float32))
+    return float(-np.sum(nz * np.log(nz)))
 
 
 def route(cat_logits, code_index: int, L_ctx: int, tau: float = TAU):
     """(category, entropy, model, pld) for one request."""
-    l = np.asarray(cat_logits, dtype=np.float32)
+    l = np.asarray(cat_logits, dtype=np.float64)
     c = int(np.argmax(l))
     H = entropy(l)
     code = c == code_index
-    model = MODEL_1B if (code and L_ctx <= SHORT_CONTEXT and H <= np.float32(tau)) else MODEL_7B
+    model = MODEL_1B if (code and L_ctx <= SHORT_CONTEXT and H <= float(tau)) else MODEL_7B
     return c, H, model, (not code)

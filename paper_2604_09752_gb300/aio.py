@@ -42,7 +42,7 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
-AIO_ABI_VERSION = 5
+AIO_ABI_VERSION = 6
 AIO_X_GIVEN = 0
 AIO_X_RMSNORM = 1
 AIO_X_SWIGLU = 2
@@ -92,6 +92,7 @@ _SIGS = {
     "aio_decode_step_create_chained": (_int, [ctypes.POINTER(_vp), ctypes.POINTER(aio_proj),
                                               ctypes.POINTER(aio_xprep), _int, _int, _u]),
     "aio_decode_step": (_int, [_vp, _vp]),
+    "aio_decode_step_host": (_int, [_vp, _vp, _vp, _sz, _vp, _vp, _sz, _vp]),
     "aio_decode_step_kernels": (_int, [_vp, ctypes.POINTER(_int)]),
     "aio_decode_step_check": (_int, [_vp, ctypes.POINTER(_int)]),
     "aio_decode_step_reset": (_int, [_vp]),
@@ -205,6 +206,12 @@ def aio_decode_step_create_chained(projs, preps, M: int, flags: int = AIO_STEP_G
 
 def aio_decode_step(step: int, stream: int = 0):
     _check(_lib.aio_decode_step(step, stream), "aio_decode_step")
+
+
+def aio_decode_step_host(step: int, x_host: int, x_dev: int, x_bytes: int, y_dev: int, y_host: int, y_bytes: int,
+                         stream: int = 0):
+    _check(_lib.aio_decode_step_host(step, x_host, x_dev, x_bytes, y_dev, y_host, y_bytes, stream),
+           "aio_decode_step_host")
 
 
 def aio_decode_step_kernels(step: int) -> int:

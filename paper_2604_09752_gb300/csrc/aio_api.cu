@@ -140,27 +140,35 @@ aio_status valid_linear(aio_linear_t h) {
     return AIO_OK;
 }
 
-aio::ProjDesc make_desc(const aio_linear* h, const void* x, const void* W, const void* scales, float* y,
-                        float* partial) {
+// The descriptor of one projection with weights W [N, K] streamed over geometry geo: the one
+// construction behind aio_linear_run, the decode steps and aio_linear_run_noalloc.
+aio::ProjDesc make_desc_geo(const aio::Geometry& geo, int K, int N, bool rowmajor, const void* x, const void* W,
+                            const void* scales, float* y, float* partial) {
     aio::ProjDesc d = {};
     d.x = static_cast<const uint16_t*>(x);
     d.w = static_cast<const uint8_t*>(W);
     d.scales = static_cast<const uint16_t*>(scales);
     d.y = y;
     d.partial = partial;
-    d.T = h->geo.T;
-    d.Tq = static_cast<int>(h->geo.T / h->geo.Z);
-    d.Tr = static_cast<int>(h->geo.T % h->geo.Z);
-    d.K = h->K;
-    d.N = h->N;
-    d.NG = h->geo.NG;
-    d.NKT = h->geo.NKT;
-    d.rowmajor = (h->flags & AIO_FLAG_ROWMAJOR) ? 1 : 0;
-    d.uniform = (!d.rowmajor && h->N % aio::kRows == 0 && h->K % aio::kKT == 0) ? 1 : 0;
+    d.T = geo.T;
+    d.Tq = static_cast<int>(geo.T / geo.Z);
+    d.Tr = static_cast<int>(geo.T % geo.Z);
+    d.K = K;
+    d.N = N;
+    d.NG = geo.NG;
+    d.NKT = geo.NKT;
+    d.rowmajor = rowmajor ? 1 : 0;
+    d.uniform = (!rowmajor && N % aio::kRows == 0 && K % aio::kKT == 0) ? 1 : 0;
     return d;
 }
 
-aio::StreamArgs single_args(const aio_linear* h, const aio::ProjDesc& d, int M, int* err) {
+aio::ProjDesc make_desc(const aio_linear* h, const void* x, const void* W, const void* scales, float* y,
+                        float* partial) {
+    return make_desc_geo(h->geo, h->K, h->N, (h->flags & AIO_FLAG_ROWMAJOR) != 0, x, W, scales, y, partial);
+}
+
+// Launch arguments of a single-projection launch (no grid barrier, no done counters).
+aio::StreamArgs single_args_geo(const aio::ProjDesc& d, int Z, int M, int* err, bool test_stall) {
     aio::StreamArgs a = {};
     a.projs = nullptr;
     a.one = d;
@@ -169,24 +177,41 @@ aio::StreamArgs single_args(const aio_linear* h, const aio::ProjDesc& d, int M, 
     a.err = err;
     a.nproj = 1;
     a.M = M;
-    a.Z = h->geo.Z;
-    a.test_stall = (h->flags & AIO_FLAG_TEST_STALL) ? 1 : 0;
-    a.wait_limit_ns = a.test_stall ? kTestWaitLimitNs : kWaitLimitNs;
+    a.Z = Z;
+    a.test_stall = test_stall ? 1 : 0;
+    a.wait_limit_ns = test_stall ? kTestWaitLimitNs : kWaitLimitNs;
     return a;
 }
 
-aio_status validate_run(const aio_linear* h, const void* x, int M, const void* W, const void* scales, const float* y) {
-    if (M < 1 || M > h->max_M) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, max_M=%d]", M, h->max_M);
+aio::StreamArgs single_args(const aio_linear* h, const aio::ProjDesc& d, int M, int* err) {
+    return single_args_geo(d, h->geo.Z, M, err, (h->flags & AIO_FLAG_TEST_STALL) != 0);
+}
+
+// Shape and weight-type checks shared by aio_linear_create and aio_linear_run_noalloc.
+aio_status validate_shape(int K, int N, aio_wtype wt) {
+    if (K < 16 || K > (1 << 20) || K % 16 != 0) return fail(AIO_ERR_INVALID_ARG, "K=%d: need 16 <= K <= 2^20, K %% 16 == 0", K);
+    if (N < 1 || N > (1 << 24)) return fail(AIO_ERR_INVALID_ARG, "N=%d: need 1 <= N <= 2^24", N);
+    if (wt != AIO_W_BF16 && wt != AIO_W_INT8_PERCHANNEL) return fail(AIO_ERR_INVALID_ARG, "unknown weight type %d", (int)wt);
+    return AIO_OK;
+}
+
+// Pointer checks of a run, shared by aio_linear_run, the decode steps and aio_linear_run_noalloc.
+aio_status validate_io(aio_wtype wt, const void* x, const void* W, const void* scales, const float* y) {
     if (!x || !W || !y) return fail(AIO_ERR_INVALID_ARG, "x, W and y must be non-NULL");
     if (!aligned(x, 16) || !aligned(W, 16) || !aligned(y, 16))
         return fail(AIO_ERR_ALIGNMENT, "x, W and y must be 16-byte aligned");
-    if (h->wt == AIO_W_INT8_PERCHANNEL) {
+    if (wt == AIO_W_INT8_PERCHANNEL) {
         if (!scales) return fail(AIO_ERR_INVALID_ARG, "int8 weights need per-channel scales");
         if (!aligned(scales, 2)) return fail(AIO_ERR_ALIGNMENT, "scales must be 2-byte aligned");
     } else if (scales) {
         return fail(AIO_ERR_INVALID_ARG, "bf16 weights take no scales (pass NULL)");
     }
     return AIO_OK;
+}
+
+aio_status validate_run(const aio_linear* h, const void* x, int M, const void* W, const void* scales, const float* y) {
+    if (M < 1 || M > h->max_M) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, max_M=%d]", M, h->max_M);
+    return validate_io(h->wt, x, W, scales, y);
 }
 
 }  // namespace
@@ -214,9 +239,10 @@ const char* aio_last_error(void) { return g_last_error; }
 aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int max_M, unsigned flags) {
     if (!out) return fail(AIO_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
-    if (K < 16 || K > (1 << 20) || K % 16 != 0) return fail(AIO_ERR_INVALID_ARG, "K=%d: need 16 <= K <= 2^20, K %% 16 == 0", K);
-    if (N < 1 || N > (1 << 24)) return fail(AIO_ERR_INVALID_ARG, "N=%d: need 1 <= N <= 2^24", N);
-    if (wt != AIO_W_BF16 && wt != AIO_W_INT8_PERCHANNEL) return fail(AIO_ERR_INVALID_ARG, "unknown weight type %d", (int)wt);
+    {
+        const aio_status sv = validate_shape(K, N, wt);
+        if (sv != AIO_OK) return sv;
+    }
     if (max_M < 1 || max_M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "max_M=%d outside [1, 8]", max_M);
     if (flags & ~kCreateFlags) return fail(AIO_ERR_INVALID_ARG, "unknown flags 0x%x", flags & ~kCreateFlags);
     int dev = 0, sms = 0;
@@ -581,6 +607,20 @@ aio_status aio_decode_step(aio_step_t s, void* stream) {
     return step_launch_all(s, static_cast<cudaStream_t>(stream));
 }
 
+aio_status aio_decode_step_host(aio_step_t s, const void* x_host, void* x_dev, size_t x_bytes, const void* y_dev,
+                                void* y_host, size_t y_bytes, void* stream) {
+    aio_status st = valid_step(s);
+    if (st != AIO_OK) return st;
+    if ((x_bytes && (!x_host || !x_dev)) || (y_bytes && (!y_host || !y_dev)))
+        return fail(AIO_ERR_INVALID_ARG, "a copy of non-zero size needs both of its pointers");
+    if ((st = check_device(s->device)) != AIO_OK) return st;
+    const cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    if (x_bytes) AIO_CUDA(cudaMemcpyAsync(x_dev, x_host, x_bytes, cudaMemcpyHostToDevice, cs));
+    if ((st = aio_decode_step(s, stream)) != AIO_OK) return st;
+    if (y_bytes) AIO_CUDA(cudaMemcpyAsync(y_host, y_dev, y_bytes, cudaMemcpyDeviceToHost, cs));
+    return AIO_OK;
+}
+
 aio_status aio_decode_step_kernels(aio_step_t s, int* n_kernels) {
     aio_status st = valid_step(s);
     if (st != AIO_OK) return st;
@@ -671,24 +711,16 @@ aio_status noalloc_scratch(int dev, void** out) {
 extern "C" aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N, aio_wtype wt, unsigned flags,
                                              const void* W, const void* scales, float* y, int* device_error,
                                              void* stream) {
-    if (K < 16 || K > (1 << 20) || K % 16 != 0) return fail(AIO_ERR_INVALID_ARG, "K=%d: need 16 <= K <= 2^20, K %% 16 == 0", K);
-    if (N < 1 || N > (1 << 24)) return fail(AIO_ERR_INVALID_ARG, "N=%d: need 1 <= N <= 2^24", N);
-    if (wt != AIO_W_BF16 && wt != AIO_W_INT8_PERCHANNEL) return fail(AIO_ERR_INVALID_ARG, "unknown weight type %d", (int)wt);
+    aio_status st = validate_shape(K, N, wt);
+    if (st != AIO_OK) return st;
     if (M < 1 || M > aio::kMaxM) return fail(AIO_ERR_INVALID_ARG, "M=%d outside [1, 8]", M);
     const unsigned allowed = AIO_FLAG_ROWMAJOR | AIO_FLAG_NO_PDL;
     if (flags & ~allowed) return fail(AIO_ERR_INVALID_ARG, "unknown flags 0x%x (ROWMAJOR and NO_PDL only)", flags & ~allowed);
-    if (!x || !W || !y || !device_error) return fail(AIO_ERR_INVALID_ARG, "x, W, y and device_error must be non-NULL");
-    if (!aligned(x, 16) || !aligned(W, 16) || !aligned(y, 16))
-        return fail(AIO_ERR_ALIGNMENT, "x, W and y must be 16-byte aligned");
+    if (!device_error) return fail(AIO_ERR_INVALID_ARG, "device_error must be non-NULL");
+    if ((st = validate_io(wt, x, W, scales, y)) != AIO_OK) return st;
     if (!aligned(device_error, 4)) return fail(AIO_ERR_ALIGNMENT, "device_error must be 4-byte aligned");
-    if (wt == AIO_W_INT8_PERCHANNEL) {
-        if (!scales) return fail(AIO_ERR_INVALID_ARG, "int8 weights need per-channel scales");
-        if (!aligned(scales, 2)) return fail(AIO_ERR_ALIGNMENT, "scales must be 2-byte aligned");
-    } else if (scales) {
-        return fail(AIO_ERR_INVALID_ARG, "bf16 weights take no scales (pass NULL)");
-    }
     int dev = 0, sms = 0;
-    aio_status st = current_device(&dev, &sms);
+    st = current_device(&dev, &sms);
     if (st != AIO_OK) return st;
     const aio::Geometry geo = aio::geometry(K, N, sms);
     const size_t need = aio::workspace_bytes(geo, M);
@@ -706,30 +738,8 @@ extern "C" aio_status aio_linear_run_noalloc(const void* x, int M, int K, int N,
     // The partial-sum slots must start empty (all bytes 0xFF); a healthy run leaves them so, an
     // expired wait may not, and the array starts out zeroed.
     AIO_CUDA(cudaMemsetAsync(partial, 0xFF, need, s));
-    aio::ProjDesc d = {};
-    d.x = static_cast<const uint16_t*>(x);
-    d.w = static_cast<const uint8_t*>(W);
-    d.scales = static_cast<const uint16_t*>(scales);
-    d.y = y;
-    d.partial = partial;
-    d.T = geo.T;
-    d.Tq = static_cast<int>(geo.T / geo.Z);
-    d.Tr = static_cast<int>(geo.T % geo.Z);
-    d.K = K;
-    d.N = N;
-    d.NG = geo.NG;
-    d.NKT = geo.NKT;
-    d.rowmajor = (flags & AIO_FLAG_ROWMAJOR) ? 1 : 0;
-    d.uniform = (!d.rowmajor && N % aio::kRows == 0 && K % aio::kKT == 0) ? 1 : 0;
-    aio::StreamArgs a = {};
-    a.projs = nullptr;
-    a.one = d;
-    a.err = device_error;
-    a.nproj = 1;
-    a.M = M;
-    a.Z = geo.Z;
-    a.test_stall = 0;
-    a.wait_limit_ns = kWaitLimitNs;
+    const aio::ProjDesc d = make_desc_geo(geo, K, N, (flags & AIO_FLAG_ROWMAJOR) != 0, x, W, scales, y, partial);
+    const aio::StreamArgs a = single_args_geo(d, geo.Z, M, device_error, false);
     AIO_CUDA(aio::launch_stream(a, wt == AIO_W_INT8_PERCHANNEL, geo.grid, s, !(flags & AIO_FLAG_NO_PDL), false));
     return AIO_OK;
 }

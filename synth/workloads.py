@@ -83,7 +83,9 @@ class Workload:
                         self.description)
 
 
-def _decoder(layers: int, H: int, I: int, qkv: int, vocab: int) -> List[Proj]:
+def decoder(layers: int, H: int, I: int, qkv: int, vocab: int) -> List[Proj]:
+    """The projections of a decoder in step order: per layer QKV (H -> qkv), O (H -> H), gate+up
+    (H -> 2I), down (I -> H), then the lm_head (H -> vocab)."""
     projs = []
     for l in range(layers):
         projs.append(Proj(l, 0, H, qkv))
@@ -100,15 +102,15 @@ def _build():
         "linear-2048", 0, "bf16", 1, [Proj(0, 1, 2048, 2048)],
         "single linear y = x W^T, M=1, K=N=2048, bf16 (8 MB of weights)")
     w["1b-bf16"] = Workload(
-        "1b-bf16", 1, "bf16", 1, _decoder(22, 2048, 5632, 6144, 32000),
+        "1b-bf16", 1, "bf16", 1, decoder(22, 2048, 5632, 6144, 32000),
         "1B-class decode step, M=1, bf16: 22 layers, hidden 2048, QKV 2048->6144, O 2048->2048, "
         "gate+up 2048->11264, down 5632->2048, lm_head 2048->32000")
     w["7b-bf16"] = Workload(
-        "7b-bf16", 7, "bf16", 1, _decoder(32, 4096, 11008, 12288, 32000),
+        "7b-bf16", 7, "bf16", 1, decoder(32, 4096, 11008, 12288, 32000),
         "7B-class decode step, M=1, bf16: 32 layers, hidden 4096, QKV 4096->12288, O 4096->4096, "
         "gate+up 4096->22016, down 11008->4096, lm_head 4096->32000")
     w["7b-int8"] = Workload(
-        "7b-int8", 7, "int8", 1, _decoder(32, 4096, 11008, 12288, 32000),
+        "7b-int8", 7, "int8", 1, decoder(32, 4096, 11008, 12288, 32000),
         "7B-class decode step, M=1, int8 weight-only codes with per-output-channel bf16 scales")
     return w
 

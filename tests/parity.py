@@ -22,12 +22,22 @@ def abs_bits(h: np.ndarray) -> np.ndarray:
     return h & np.uint16(0x7FFF)
 
 
+def abs_codes(q: np.ndarray):
+    """|q| as int8 operands of the oracle: |q| = lo + hi with lo = min(|q|, 127) and hi = 1 exactly
+    where q = -128 (|-128| = 128 does not fit int8)."""
+    a = np.abs(q.astype(np.int16))
+    return np.minimum(a, 127).astype(np.int8), (a == 128).astype(np.int8)
+
+
 def reference(x: np.ndarray, W: np.ndarray, s=None):
     """(y_ref, sum |x_k w_k|) from the oracle; x [M, K] uint16, W [N, K] uint16 or int8."""
     if W.dtype == np.int8:
         y = oracle.linear_i8(x, W, s)
-        qa = np.abs(W.astype(np.int16)).astype(np.int8)   # |q| <= 127 fits
-        mag = oracle.linear_i8(abs_bits(x), qa, s)
+        lo, hi = abs_codes(W)
+        xa = abs_bits(x)
+        mag = oracle.linear_i8(xa, lo, s)
+        if hi.any():
+            mag = mag + oracle.linear_i8(xa, hi, s)
     else:
         y = oracle.linear_bf16(x, W)
         mag = oracle.linear_bf16(abs_bits(x), abs_bits(W))

@@ -99,10 +99,22 @@ def teacher_forced(dw, M, what, rows_of=None):
     return ys
 
 
-@pytest.mark.parametrize("name,M", [("1b-bf16", 1), ("1b-bf16", 2), ("1b-bf16", 3), ("7b-int8", 1), ("7b-bf16", 1)])
+def narrow_chain(wtype):
+    """Two layers of a decoder with hidden 2048 and intermediate 2048 (QKV 6144, vocabulary 4096):
+    every computed x fits the staging area at M = 4, which the 1B and 7B down projections (K = 5632,
+    11008) do not."""
+    return swl.Workload(f"narrow-{wtype}", 2, wtype, 1, swl.decoder(2, 2048, 2048, 6144, 4096),
+                        "two-layer narrow decoder for chained M = 4")
+
+
+@pytest.mark.parametrize("name,M", [("1b-bf16", 1), ("1b-bf16", 2), ("1b-bf16", 3), ("7b-int8", 1), ("7b-bf16", 1),
+                                    ("narrow-bf16", 4), ("narrow-int8", 4), ("narrow-bf16", 3)])
 def test_small_chain(aio, name, M):
     from paper_2604_09752_gb300.workload import DeviceWorkload
-    wl = swl.truncated(swl.WORKLOADS[name], 2)
+    if name.startswith("narrow-"):
+        wl = narrow_chain(name.split("-")[1])
+    else:
+        wl = swl.truncated(swl.WORKLOADS[name], 2)
     dw = DeviceWorkload(wl, seed=3, max_M=M, chained=True)
     dw.fill_chain(M)
     dw.x_arena.fill_(0xFF)

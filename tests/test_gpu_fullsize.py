@@ -44,7 +44,7 @@ def test_full_7b_step_sampled(aio, name):
     rng = np.random.default_rng(0)
     dw = DeviceWorkload(swl.WORKLOADS[name], seed=0, max_M=8)
     flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
-    for M in (1, 8):
+    for M in (1, 4, 8):   # M = 4 and 8 at K = 11008 read x unstaged
         dw.fill_x(M)
         dw.y_arena.fill_(0xFF)                      # NaN everywhere: every output must be written
         for _ in range(3):

@@ -1,5 +1,7 @@
 """GPU parity of one linear layer through the C ABI: y = x W^T (Sec. 2.1), int8 with per-channel
-scales (Sec. 2.4), M = 1..8 token rows (Sec. 4.2), packed and row-major weights, ragged shapes."""
+scales (Sec. 2.4), every width M = 1..8 the API accepts (Sec. 4.2 verification rows), packed and
+row-major weights, ragged shapes, and the int8 code -128 (outside the symmetric range the recipe
+draws, but a valid code the kernel must convert exactly)."""
 import numpy as np
 import pytest
 import torch
@@ -65,7 +67,7 @@ SHAPES = [(16, 1), (48, 13), (272, 9), (1040, 37), (2048, 2048), (4096, 100), (5
 
 @pytest.mark.parametrize("wt", ["bf16", "int8"])
 @pytest.mark.parametrize("K,N", SHAPES)
-@pytest.mark.parametrize("M", [1, 2, 3, 8])
+@pytest.mark.parametrize("M", [1, 2, 3, 4, 5, 6, 7, 8])
 @pytest.mark.parametrize("layout_", ["packed", "rowmajor"])
 def test_linear_parity(aio, wt, K, N, M, layout_):
     x, W, s = make_inputs(K, N, M, wt)
@@ -131,6 +133,54 @@ def test_int8_known_codes_exact(aio):
     torch.cuda.synchronize()
     assert y.cpu().numpy().tolist() == [-0.9921875, np.float32(0.0050048828125 * 127)]
     lin.close()
+
+
+@pytest.mark.parametrize("K,N,layout_", [(16, 3, "packed"), (4096, 64, "packed"), (1040, 37, "packed"),
+                                         (4096, 64, "rowmajor")])
+def test_int8_code_minus_128_one_hot_exact(aio, K, N, layout_):
+    """q = -128 in the columns the one-hot x rows select (full, ragged and row-major tiles), a few bf16
+    scales: y[m, n] = s[n] * -128 exactly (s * 2^7 is exact in fp32 and in the oracle's double)."""
+    ks = [0, 1, 255, 256, K - 1] if K > 256 else [0, 3, K - 1]
+    q = synth.codes_i8(synth.key(21, K, N), N * K).reshape(N, K)
+    q[:, ks] = -128
+    # a few bf16 scales: 2^-7, bf16(0.005), the smallest and largest of the recipe's range
+    s = np.resize(np.array([0x3C00, 0x3BA4, 0x3A83, 0x3C24], np.uint16), N)
+    x = np.zeros((len(ks), K), np.uint16)
+    for m, k in enumerate(ks):
+        x[m, k] = 0x3F80
+    lin = Linear(aio, q, s, max_M=8, rowmajor=(layout_ == "rowmajor"))
+    y = torch.empty(len(ks) * N, dtype=torch.float32, device="cuda")
+    lin.run(dev(x), len(ks), y)
+    torch.cuda.synchronize()
+    got = y.cpu().numpy().reshape(len(ks), N)
+    want = (s.astype(np.uint32) << 16).view(np.float32) * np.float32(-128.0)
+    assert np.array_equal(got, np.broadcast_to(want, got.shape))
+    y_ref, _ = parity.reference(x, q, s)
+    assert np.array_equal(got.astype(np.float64), y_ref)
+    lin.close()
+
+
+@pytest.mark.parametrize("K,N", [(4096, 64), (1040, 37), (11008, 40)])
+@pytest.mark.parametrize("M", [1, 4, 8])
+def test_int8_rows_of_minus_128_and_full_code_range(aio, K, N, M):
+    """Whole rows of -128 (every second row group's first row, and the last row) inside weights that
+    take every int8 code in [-128, 127], against the fp64 oracle at the stated bar."""
+    x, _, s = make_inputs(K, N, M, "int8", tag=23)
+    u = synth.codes_i8(synth.key(23, K, N, 9), N * K).astype(np.int16).reshape(N, K)
+    # every int8 code: 127 stays at odd k and becomes -128 at even k
+    q = np.where((u == 127) & (np.arange(K) % 2 == 0), -128, u).astype(np.int8)
+    q[0::32] = -128
+    q[N - 1] = -128
+    assert (q == -128).any(axis=1).sum() >= 2 and (q == -128).sum() > N
+    for rowmajor in (False, True):
+        lin = Linear(aio, q, s, max_M=8, rowmajor=rowmajor)
+        y = torch.full((M * N,), float("nan"), dtype=torch.float32, device="cuda")
+        lin.run(dev(x), M, y)
+        torch.cuda.synchronize()
+        assert aio.aio_linear_check(lin.h) == 0
+        y_ref, mag = parity.reference(x, q, s)
+        parity.check(y.cpu().numpy().reshape(M, N), y_ref, mag, K, f"-128 K={K} N={N} M={M} rowmajor={rowmajor}")
+        lin.close()
 
 
 def test_deterministic_and_repeatable(aio):

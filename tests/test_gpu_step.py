@@ -39,7 +39,7 @@ def check_workload(dw, M, what):
 
 
 @pytest.mark.parametrize("name", ["1b-bf16", "7b-int8"])
-@pytest.mark.parametrize("M", [1, 3, 8])
+@pytest.mark.parametrize("M", [1, 3, 4, 8])
 def test_small_step_graph_pdl(aio, name, M):
     from paper_2604_09752_gb300.workload import DeviceWorkload
     dw = DeviceWorkload(swl.WORKLOADS[name], seed=1, max_M=8, projs=small_decoder(name))
@@ -49,6 +49,28 @@ def test_small_step_graph_pdl(aio, name, M):
     assert aio.aio_decode_step_kernels(dw.step_handle(M, aio.AIO_STEP_PDL)) == len(dw.bufs)
     assert aio.aio_decode_step_check(dw.step_handle(M)) == 0
     check_workload(dw, M, f"{name} M={M}")
+    dw.close()
+
+
+def test_step_from_host_buffers(aio):
+    """aio_decode_step_host: x copied in from pinned host memory, the step, y copied back, in stream
+    order; the host y equals the device y, and both meet the bar against the oracle."""
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    dw = DeviceWorkload(swl.WORKLOADS["7b-int8"], seed=6, max_M=2, projs=small_decoder("7b-int8", 1))
+    x_host = dw.fill_x(2)
+    dw.x_arena.zero_()
+    dw.y_arena.fill_(0xFF)
+    y_host = torch.full((dw.y_arena.numel(),), 0xAB, dtype=torch.uint8).pin_memory()
+    s = torch.cuda.current_stream().cuda_stream
+    aio.aio_decode_step_host(dw.step_handle(2), x_host.data_ptr(), dw.x_arena.data_ptr(), x_host.numel(),
+                             dw.y_arena.data_ptr(), y_host.data_ptr(), y_host.numel(), s)
+    torch.cuda.synchronize()
+    assert aio.aio_decode_step_check(dw.step_handle(2)) == 0
+    assert torch.equal(y_host, dw.y_arena.cpu())
+    check_workload(dw, 2, "from host buffers")
+    with pytest.raises(aio.AioError) as e:
+        aio.aio_decode_step_host(dw.step_handle(2), None, dw.x_arena.data_ptr(), 16, 0, 0, 0, s)
+    assert e.value.status == aio.AIO_ERR_INVALID_ARG
     dw.close()
 
 

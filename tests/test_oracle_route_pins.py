@@ -12,11 +12,17 @@ CODE, QA, MATH = 0, 1, 2
 
 
 def test_entropy_closed_forms():
-    assert abs(route.entropy([0.0, 0.0, 0.0]) - math.log(3)) < 1e-6          # uniform: ln n
-    assert route.entropy([0.0, -200.0, -200.0]) < 1e-6                        # one certain category
+    # the oracle evaluates the definition in double: closed forms hold to a few double ulps
+    assert abs(route.entropy([0.0, 0.0, 0.0]) - math.log(3)) < 1e-15          # uniform: ln n
+    assert abs(route.entropy([0.0] * 32) - math.log(32)) < 1e-14
+    assert route.entropy([0.0, -200.0, -200.0]) < 1e-80                       # one certain category
     h = route.entropy([math.log(3), 0.0])                                     # p = (3/4, 1/4)
-    assert abs(h - (-(0.75 * math.log(0.75) + 0.25 * math.log(0.25)))) < 1e-6
-    assert abs(route.entropy([5.0, 5.0, 5.0]) - route.entropy([0.0, 0.0, 0.0])) < 1e-6   # shift invariant
+    assert abs(h - (-(0.75 * math.log(0.75) + 0.25 * math.log(0.25)))) < 1e-15
+    assert route.entropy([5.0, 5.0, 5.0]) == route.entropy([0.0, 0.0, 0.0])   # shift invariant
+    # two categories with logit gap g: p = 1 / (1 + e^-g), H = ln(1 + e^-g) + g e^-g / (1 + e^-g)
+    for g in (0.5, 2.0, 2.7, 9.0):
+        eg = math.exp(-g)
+        assert abs(route.entropy([g, 0.0]) - (math.log1p(eg) + g * eg / (1 + eg))) < 1e-15
 
 
 def test_decision_table():
