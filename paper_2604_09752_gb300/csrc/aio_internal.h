@@ -38,6 +38,15 @@
 #ifndef AIO_SLOT_KB_I8
 #define AIO_SLOT_KB_I8 AIO_SLOT_KB   // the same for int8 weights (4 KB tiles)
 #endif
+// Launches with M >= AIO_WIDE_M token rows use a ring of AIO_RING_KB_WIDE per warp instead, so that
+// the area left for staged x holds M rows of the 4096-column projections (and M <= 4 rows of
+// K = 11008 would fit it too): at such widths a tile's x read from L2 costs more than a ring slot.
+#ifndef AIO_RING_KB_WIDE
+#define AIO_RING_KB_WIDE 16
+#endif
+#ifndef AIO_WIDE_M
+#define AIO_WIDE_M 5
+#endif
 
 namespace aio {
 
@@ -45,24 +54,39 @@ constexpr int kRows = 16;                   // rows per row group (AIO_ROWS_PER_
 constexpr int kKT = 256;                    // k columns per tile (AIO_K_TILE)
 constexpr int kWarps = AIO_WARPS;           // every warp streams its own tile segment
 constexpr int kThreads = kWarps * 32;
-constexpr int kRingBytesPerWarp = AIO_RING_KB * 1024;
 constexpr int kSlotBytes = AIO_SLOT_KB * 1024;
-constexpr int kStages = kRingBytesPerWarp / kSlotBytes;  // ring slots per warp
 constexpr int kSlotBytesI8 = AIO_SLOT_KB_I8 * 1024;
-constexpr int kStagesI8 = kRingBytesPerWarp / kSlotBytesI8;
-constexpr int kMaxStages = kStages > kStagesI8 ? kStages : kStagesI8;
-static_assert(kSlotBytes % 8192 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
-static_assert(kSlotBytesI8 % 4096 == 0 && kStagesI8 >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
-constexpr int kSyncOffset = kWarps * kRingBytesPerWarp + kWarps * kMaxStages * 8;  // CTA-level sync words
 constexpr int kMaxM = 8;
-constexpr int kAuxOffset = kSyncOffset + 32;       // sync words (16 B), the x barrier (8 B), padding
-constexpr int kAuxBytes = kWarps * kMaxM * 4;      // per-warp, per-token partial sums (x preparation)
-constexpr int kXsOffset = kAuxOffset + (kAuxBytes + 15) / 16 * 16;
 constexpr int kXsPad = 32;                         // elements between staged x rows beyond K (64 B)
-constexpr int kXsBytes = 227 * 1024 - kXsOffset;   // x staged in shared memory when M * (K + kXsPad) * 2 fits
-constexpr int kSmemBytes = kXsOffset + kXsBytes;
-static_assert(kSmemBytes <= 227 * 1024, "ring does not fit in shared memory");
-static_assert(kXsOffset % 16 == 0, "bulk-copy destination alignment");
+constexpr int kSmemBytes = 227 * 1024;             // dynamic shared memory of every stream-kernel launch
+
+// Shared memory of one CTA with a ring of RingKB per warp: the warps' rings, their slot barriers,
+// CTA sync words and the x barrier, x-preparation scratch, then the staged x in the rest.
+template <int RingKB>
+struct SmemLayout {
+    static constexpr int kRingBytes = RingKB * 1024;                 // per warp
+    static constexpr int kStages = kRingBytes / kSlotBytes;          // bf16 ring slots per warp
+    static constexpr int kStagesI8 = kRingBytes / kSlotBytesI8;      // int8 ring slots per warp
+    static constexpr int kMaxStages = kStages > kStagesI8 ? kStages : kStagesI8;
+    static constexpr int kSyncOffset = kWarps * kRingBytes + kWarps * kMaxStages * 8;   // CTA-level sync words
+    static constexpr int kAuxOffset = kSyncOffset + 32;  // sync words (16 B), the x barrier (8 B), padding
+    static constexpr int kAuxBytes = kWarps * kMaxM * 4; // per-warp, per-token partial sums (x preparation)
+    static constexpr int kXsOffset = kAuxOffset + (kAuxBytes + 15) / 16 * 16;
+    static constexpr int kXsBytes = kSmemBytes - kXsOffset;  // x staged when M * (K + kXsPad) * 2 fits
+    static_assert(kSlotBytes % 8192 == 0 && kStages >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
+    static_assert(kSlotBytesI8 % 4096 == 0 && kStagesI8 >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
+    static_assert(kXsOffset % 16 == 0 && kXsBytes > 0, "ring does not fit in shared memory");
+};
+using NarrowLayout = SmemLayout<AIO_RING_KB>;       // launches of M < AIO_WIDE_M token rows
+using WideLayout = SmemLayout<AIO_RING_KB_WIDE>;    // M >= AIO_WIDE_M
+template <int MT>
+using LayoutFor = SmemLayout<(MT >= AIO_WIDE_M ? AIO_RING_KB_WIDE : AIO_RING_KB)>;
+// The narrow layout's values, for code that runs at every width (the read probe, attention) and for
+// the chained step, whose kernels exist for M <= 4 only.
+constexpr int kRingBytesPerWarp = NarrowLayout::kRingBytes;
+constexpr int kStages = NarrowLayout::kStages;
+constexpr int kMaxStages = NarrowLayout::kMaxStages;
+constexpr int kXsBytes = NarrowLayout::kXsBytes;
 
 constexpr int kDevErrTimeout = 1;       // a bulk-copy wait expired
 constexpr int kDevErrGridTimeout = 2;   // a wait for the previous projection expired
@@ -129,6 +153,7 @@ cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared 
 // pdl: programmatic dependent launch; coop: cooperative launch (all CTAs co-resident).
 using StreamFn = void (*)(const StreamArgs);
 constexpr int kMaxChainM = 4;   // token rows of a chained step (its kernels are instantiated for M <= 4)
+static_assert(kMaxChainM < AIO_WIDE_M, "the chained step's staging limit is the narrow layout's");
 StreamFn chain_stream_fn(bool i8, int M);   // aio_chain.cu
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop,
                           bool chained = false);

@@ -208,7 +208,6 @@ struct TileT {
     static constexpr int kEsize = I8 ? 1 : 2;
     static constexpr int kBytes = kRows * kKT * kEsize;    // 4096 (int8) or 8192 (bf16)
     static constexpr int kSlot = I8 ? kSlotBytesI8 : kSlotBytes;
-    static constexpr int kStagesT = I8 ? kStagesI8 : kStages;   // ring slots per warp
     static constexpr int kChunk = kSlot / kBytes;          // tiles per ring slot
     static constexpr int kAhead = I8 ? AIO_AHEAD_I8 : AIO_AHEAD;
     static constexpr int kAheadLive = I8 ? AIO_AHEAD_LIVE_I8 : AIO_AHEAD_LIVE;
@@ -1032,21 +1031,22 @@ __device__ __forceinline__ void prep_x(const ProjDesc* d, uint16_t* xs, int xs_s
 template <int MT, bool I8, bool CH>
 __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_constant__ StreamArgs s) {
     using TL = TileT<I8>;
+    using SL = LayoutFor<MT>;
     constexpr int C = TL::kChunk;
-    constexpr int S = TL::kStagesT;
+    constexpr int S = I8 ? SL::kStagesI8 : SL::kStages;   // ring slots per warp
     constexpr int E = TL::kEsize;
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    uint8_t* ring = smem + warp * kRingBytesPerWarp;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kRingBytesPerWarp) + warp * kMaxStages;
+    uint8_t* ring = smem + warp * SL::kRingBytes;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * SL::kRingBytes) + warp * SL::kMaxStages;
     // CTA-level sync words: [0] warps of this CTA done with the current phase, [1] highest projection
     // index whose predecessor is known complete (published by warp 0).
-    unsigned* cta_sync = reinterpret_cast<unsigned*>(smem + kSyncOffset);
+    unsigned* cta_sync = reinterpret_cast<unsigned*>(smem + SL::kSyncOffset);
     // x of the current projection, staged once per CTA when it fits (one bulk copy by warp 0).
-    uint64_t* xbar = reinterpret_cast<uint64_t*>(smem + kSyncOffset + 16);
-    uint16_t* xs = reinterpret_cast<uint16_t*>(smem + kXsOffset);
-    [[maybe_unused]] float* red = reinterpret_cast<float*>(smem + kAuxOffset);   // x preparation scratch
+    uint64_t* xbar = reinterpret_cast<uint64_t*>(smem + SL::kSyncOffset + 16);
+    uint16_t* xs = reinterpret_cast<uint16_t*>(smem + SL::kXsOffset);
+    [[maybe_unused]] float* red = reinterpret_cast<float*>(smem + SL::kAuxOffset);   // x preparation scratch
 
     griddep_launch_dependents();
 
@@ -1119,7 +1119,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         // Staged x rows are kXsPad elements apart beyond K, so two tokens read in one shared-memory
         // phase fall in different banks.
         const int xs_stride = P.K + kXsPad;
-        const bool stage = P.M * xs_stride * 2 <= kXsBytes;
+        const bool stage = P.M * xs_stride * 2 <= SL::kXsBytes;
         // Warp 0 stages x once every CTA has finished the previous projection (every warp of this
         // CTA has then finished reading the previous x and fenced its reads against async writes):
         // one bulk copy per token row.
