@@ -22,6 +22,11 @@ Functions and the passages they follow:
   * pld.draft / pld.argmax / pld.accept  prompt-lookup drafting (N = 6, L = 2,
                              Sec. 4.2) and greedy acceptance of the verification
                              pass (oracle/pld.py, plain Python).
+  * attention_link(y_qkv, kv, L_past, n_heads)
+                             the chained step's attention between QKV and O:
+                             the new tokens' k and v appended to the layer's KV
+                             cache, decode attention over it, x = bf16(out)
+                             (Sec. 3.3, Sec. 5.1: 2K and 32K contexts).
   * silu(t), rmsnorm(...), swiglu(...), slice_x(...)
                              the steps between the projections of a chained
                              decoder step; chain_step(...) runs a whole chained
@@ -191,11 +196,42 @@ class Oracle:
                                       out.ctypes.data)
         return out
 
-    def prep(self, link, ys, h, h0, gammas, eps):
+    def round_bf16(self, v):
+        """Each double of v rounded to bf16 (nearest, ties to even), as bf16 bits."""
+        v = np.asarray(v, dtype=np.float64)
+        return np.array([self.double_to_bf16(t) for t in v.ravel()], dtype=np.uint16).reshape(v.shape)
+
+    def attention_link(self, y_qkv, kv, L_past, n_heads, d=128):
+        """x of O when the new tokens attend over a KV cache (the chained step's attention link).
+        y_qkv [M, >= 3 n_heads d] fp32 is the QKV output: q, k, v are its column thirds, head h at
+        columns [h d, h d + d) of each.  kv [2, n_heads, L_max, d] bf16 bits is the layer's cache (K
+        then V) holding L_past positions.  Steps: the new tokens' k and v, rounded to bf16, are
+        written at positions L_past .. L_past + M - 1; token m attends to positions
+        j <= L_past + m (decode attention over L = L_past + M positions); x = bf16(out).
+        Returns (x [M, n_heads d] bf16 bits, the updated cache)."""
+        y = np.ascontiguousarray(y_qkv, dtype=np.float32)
+        M = y.shape[0]
+        H = n_heads * d
+        kv = np.array(kv, dtype=np.uint16, copy=True)
+        assert kv.shape[:2] == (2, n_heads) and kv.shape[3] == d and L_past + M <= kv.shape[2]
+        k_new = self.slice_x(y, H, H).reshape(M, n_heads, d)
+        v_new = self.slice_x(y, 2 * H, H).reshape(M, n_heads, d)
+        kv[0, :, L_past:L_past + M, :] = k_new.transpose(1, 0, 2)
+        kv[1, :, L_past:L_past + M, :] = v_new.transpose(1, 0, 2)
+        out = self.attention(y, kv[0], kv[1], L_past + M, M)
+        return self.round_bf16(out), kv
+
+    def prep(self, link, ys, h, h0, gammas, eps, caches=None):
         """x of one projection of a chained step from the buffers before it (``link``: a
         synth.workloads.ChainLink); returns (x, h_out or None).  ys: fp32 y of earlier projections
-        by index; h: the two residual buffers; h0: the step's input residual stream."""
-        from synth.workloads import XOP_RMSNORM, XOP_SWIGLU, XOP_SLICE
+        by index; h: the two residual buffers; h0: the step's input residual stream; caches: for
+        attention links, a dict layer -> [kv, L_past, n_heads] whose kv the link replaces with the
+        updated cache."""
+        from synth.workloads import XOP_RMSNORM, XOP_SWIGLU, XOP_SLICE, XOP_ATTENTION
+        if link.op == XOP_ATTENTION:
+            c = caches[link.layer]
+            x, c[0] = self.attention_link(ys[link.src], c[0], c[1], c[2])
+            return x, None
         if link.op == XOP_RMSNORM:
             h_in = h0 if link.h_in < 0 else h[link.h_in]
             r = None if link.src < 0 else ys[link.src]
@@ -208,14 +244,15 @@ class Oracle:
             return self.slice_x(ys[link.src], link.src_off, link.K), None
         raise ValueError(link.op)
 
-    def chain_step(self, links, weights, h0, gammas, eps):
+    def chain_step(self, links, weights, h0, gammas, eps, caches=None):
         """A whole chained decoder step in the oracle's own arithmetic: every projection's x from
         the oracle's earlier outputs, y rounded to fp32 as the CUDA path stores it.  weights[i] is
-        W (bf16 bits) or (q, s) for int8.  Returns (xs, ys, h) with ys in fp32."""
+        W (bf16 bits) or (q, s) for int8; caches as for prep (updated in place).  Returns
+        (xs, ys, h) with ys in fp32."""
         xs, ys = [], []
         h = [None, None]
         for link, w in zip(links, weights):
-            x, h_out = self.prep(link, ys, h, h0, gammas, eps)
+            x, h_out = self.prep(link, ys, h, h0, gammas, eps, caches)
             if h_out is not None:
                 h[link.h_out] = h_out
             y = self.linear_i8(x, *w) if isinstance(w, tuple) else self.linear_bf16(x, w)
@@ -269,8 +306,12 @@ def slice_x(y, off, K):
     return _default().slice_x(y, off, K)
 
 
-def chain_step(links, weights, h0, gammas, eps):
-    return _default().chain_step(links, weights, h0, gammas, eps)
+def chain_step(links, weights, h0, gammas, eps, caches=None):
+    return _default().chain_step(links, weights, h0, gammas, eps, caches)
+
+
+def attention_link(y_qkv, kv, L_past, n_heads, d=128):
+    return _default().attention_link(y_qkv, kv, L_past, n_heads, d)
 
 
 def attention(q, k, v, L, M=None):

@@ -22,6 +22,12 @@ Chained step (the projections wired into decoder layers, see chain_links):
                 2l + 1 (before gate+up), 2L (before lm_head)
                                            key(seed, family * 1000 + norm, 0, KIND_GAMMA)
   * RMSNorm epsilon RMS_EPS = 1e-5.
+
+Chained step with attention over a KV cache (chain_links(..., attention=True)): O takes its x from
+attention of the new tokens over layer l's cache instead of the one-position V slice.
+  * cache [2][n_heads][L_max][128] bf16 ~ N(0, 1) (K then V; positions >= L_past are overwritten by
+    the step)                              key(seed, family * 1000 + layer, 0, KIND_KV)
+  * n_heads = H / 128, the new tokens at positions L_past .. L_past + M - 1.
 """
 from __future__ import annotations
 
@@ -33,11 +39,12 @@ import numpy as np
 
 from . import codes_i8, key, normal_bf16, uniform_bf16
 
-KIND_W, KIND_X, KIND_Q, KIND_S, KIND_GAMMA, KIND_H0 = 0, 1, 2, 3, 4, 5
+KIND_W, KIND_X, KIND_Q, KIND_S, KIND_GAMMA, KIND_H0, KIND_KV = 0, 1, 2, 3, 4, 5, 6
+HEAD_DIM = 128
 RMS_EPS = 1e-5
 
 # How a projection of a chained step gets its x (the values of the C ABI's AIO_X_* constants).
-XOP_GIVEN, XOP_RMSNORM, XOP_SWIGLU, XOP_SLICE = 0, 1, 2, 3
+XOP_GIVEN, XOP_RMSNORM, XOP_SWIGLU, XOP_SLICE, XOP_ATTENTION = 0, 1, 2, 3, 4
 PROJ_NAMES = ("qkv", "o", "gate_up", "down", "lm_head")
 
 
@@ -173,7 +180,8 @@ class ChainLink:
 
     op      XOP_RMSNORM: x = RMSNorm(h_in + y[src]) with norm weight `gamma`, the sum stored in
             residual buffer h_out; XOP_SWIGLU: x = SwiGLU of y[src] (gate | up halves);
-            XOP_SLICE: x = columns [src_off, src_off + K) of y[src].
+            XOP_SLICE: x = columns [src_off, src_off + K) of y[src]; XOP_ATTENTION: x = attention
+            of the new tokens over layer `layer`'s KV cache, q, k and v the thirds of y[src].
     src     index of the projection whose y feeds x (-1: none).
     h_in    residual buffer read (-1: the step's input h0, 0 / 1: the two residual buffers).
     h_out   residual buffer written (-1: none).
@@ -185,12 +193,14 @@ class ChainLink:
     h_in: int = -1
     h_out: int = -1
     gamma: int = -1
+    layer: int = -1
 
 
-def chain_links(wl: Workload) -> List[ChainLink]:
+def chain_links(wl: Workload, attention: bool = False) -> List[ChainLink]:
     """Pre-norm decoder layers over the workload's projections (qkv, o, gate_up, down per layer,
     then lm_head).  Residual adds ride on the next RMSNorm; the two residual buffers alternate so
-    that no buffer is written while another CTA may still read it (two grid barriers apart)."""
+    that no buffer is written while another CTA may still read it (two grid barriers apart).
+    attention: O's x is attention over the layer's KV cache (else the one-position V slice)."""
     links: List[ChainLink] = []
     base = {}
     for i, p in enumerate(wl.projs):
@@ -203,6 +213,8 @@ def chain_links(wl: Workload) -> List[ChainLink]:
                 links.append(ChainLink(XOP_RMSNORM, p.K, gamma=0))
             else:
                 links.append(ChainLink(XOP_RMSNORM, p.K, src=base[(l - 1, 3)], h_in=1, h_out=0, gamma=2 * l))
+        elif p.index == 1 and attention:   # o: attention over the layer's KV cache
+            links.append(ChainLink(XOP_ATTENTION, p.K, src=base[(l, 0)], layer=l))
         elif p.index == 1:    # o: attention over one position = the V third of qkv
             q = wl.projs[base[(l, 0)]]
             links.append(ChainLink(XOP_SLICE, p.K, src=base[(l, 0)], src_off=2 * q.N // 3))
@@ -229,6 +241,16 @@ def gen_h0(seed: int, wl: Workload, M: int):
 
 def gen_gamma(seed: int, wl: Workload, norm: int, out=None):
     return uniform_bf16(key(seed, wl.family * 1000 + norm, 0, KIND_GAMMA), 0.5, 1.5, hidden(wl), 0, out)
+
+
+def n_heads(wl: Workload) -> int:
+    return hidden(wl) // HEAD_DIM
+
+
+def gen_kv_cache(seed: int, wl: Workload, layer: int, L_max: int, out=None):
+    """Layer `layer`'s KV cache [2][n_heads][L_max][128] as bf16 bits (K then V), N(0, 1)."""
+    n = 2 * n_heads(wl) * L_max * HEAD_DIM
+    return normal_bf16(key(seed, wl.family * 1000 + layer, 0, KIND_KV), 1.0, n, 0, out)
 
 
 def n_norms(wl: Workload) -> int:
