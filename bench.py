@@ -366,16 +366,29 @@ def bench_chain(args, peak):
     import torch
     flags = aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT
     out = {}
-    for name in ("7b-bf16", "7b-int8"):
+    # (workload, M, context): context None = attention over one position (O reads the V third of
+    # QKV); else attention over a KV cache of that many positions in every layer (2K, Sec. 5.1)
+    for name, M, ctx in (("7b-bf16", 1, None), ("7b-int8", 1, None), ("7b-bf16", 1, 2048), ("7b-int8", 1, 2048),
+                         ("7b-bf16", 3, 2048)):
         wl = swl.WORKLOADS[name]
-        dw = DeviceWorkload(wl, seed=args.seed, max_M=1, chained=True)
-        dw.fill_chain(1)
-        step = dw.step_handle(1, flags)
+        dw = DeviceWorkload(wl, seed=args.seed, max_M=M, chained=True, kv_len=ctx)
+        dw.fill_chain(M)
+        if ctx:
+            dw.fill_kv(ctx - M)
+        step = dw.step_handle(M, flags)
         stream = torch.cuda.Stream()
         ms = time_calls(lambda sh: aio.aio_decode_step(step, sh), stream, args.steps, args.warmup)
         assert aio.aio_decode_step_check(step) == 0
-        key = f"7b-chain-{wl.wtype}"
-        out[key] = step_record(key, 1, wl.wtype, dw.weight_bytes(), ms, peak, aio.aio_decode_step_kernels(step))
+        wbytes = dw.weight_bytes()
+        if ctx:
+            kv_bytes = len(dw.attn_layers) * 2 * dw.n_heads * ctx * swl.HEAD_DIM * 2
+            key = f"7b-chain-attn{ctx // 1024}k-{wl.wtype}" + (f"-M{M}" if M > 1 else "")
+            out[key] = step_record(key, M, wl.wtype, wbytes + kv_bytes, ms, peak, aio.aio_decode_step_kernels(step),
+                                   weight_bytes=wbytes, kv_bytes_per_step=kv_bytes, context=ctx,
+                                   note="GB/s over weight + KV-cache bytes")
+        else:
+            key = f"7b-chain-{wl.wtype}"
+            out[key] = step_record(key, M, wl.wtype, wbytes, ms, peak, aio.aio_decode_step_kernels(step))
         dw.close()
     return out
 

@@ -35,7 +35,8 @@
  *     aio_linear_check / aio_decode_step_check / aio_attention_check report as
  *     AIO_ERR_DEVICE_TIMEOUT, with the code in *device_error: 1 a bulk-copy wait expired,
  *     2 a wait for the previous projection expired, 3 a chained step's computed x did not fit
- *     the staging area (refused on the host; the device check is a second guard).
+ *     the staging area (refused on the host; the device check is a second guard), 4 a chained
+ *     step's attention found L_past + M outside [M, L_max].
  */
 #ifndef AIO_H
 #define AIO_H
@@ -47,7 +48,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 6
+#define AIO_ABI_VERSION 7
 
 typedef enum {
     AIO_OK = 0,
@@ -116,6 +117,8 @@ typedef struct {
 #define AIO_X_RMSNORM 1   /* h = h_in + src (src may be NULL), x = h * gamma / sqrt(mean(h^2) + eps) */
 #define AIO_X_SWIGLU  2   /* x[m, k] = silu(src[m, k]) * src[m, K + k], silu(t) = t / (1 + exp(-t)) */
 #define AIO_X_SLICE   3   /* x[m, k] = src[m, src_off + k] (attention over one position: V of QKV) */
+#define AIO_X_ATTENTION 4 /* x = bf16(attention of the M new tokens over the layer's KV cache), q, k, v
+                             the column thirds of src (the QKV output), see aio_xprep.kv_cache */
 
 typedef struct {
     int op;               /* AIO_X_* */
@@ -130,6 +133,21 @@ typedef struct {
                              the next grid-wide step boundary after this projection */
     const void* gamma;    /* RMSNORM: norm weight [K] bf16 */
     float eps;            /* RMSNORM: >= 0 */
+    /* ATTENTION (decode attention over a KV cache, the long-context path of Sec. 3.3 and Sec. 5.1):
+     * src is the QKV output, fp32 [M, src_stride >= 3K]; q, k and v of token m are its columns
+     * [0, K), [K, 2K) and [2K, 3K), head h at columns [128 h, 128 h + 128) of each (K = 128 n_heads).
+     * The device reads *L_past (set before the step; not changed by it), writes the new tokens' k
+     * and v, rounded to bf16, at positions L_past .. L_past + M - 1 of the cache, and computes
+     *   out[m, h] = sum_j softmax_j(q[m, h] . k[h, j] / sqrt(128)) v[h, j]  over j <= L_past + m,
+     * in fp32 with an online softmax and a fixed merge order; x = bf16(out) (nearest even).  It
+     * runs as two phases of the step before this projection, so the step grows by two grid-wide
+     * steps (two kernels in chain mode).  L_past + M > L_max is reported as device error 4 and
+     * leaves x undefined. */
+    void* kv_cache;       /* ATTENTION: the layer's cache, bf16 [2][n_heads][L_max][128] (K, then V), device,
+                             16-byte aligned; updated in place */
+    const int* L_past;    /* ATTENTION: device int, positions already in the cache, 4-byte aligned */
+    int n_heads;          /* ATTENTION: K / 128, at most the warps of the grid */
+    int L_max;            /* ATTENTION: positions the cache holds */
 } aio_xprep;
 
 /* ABI version of the loaded library (AIO_ABI_VERSION at build time). */
@@ -253,12 +271,14 @@ aio_status aio_decode_step_create(aio_step_t* out, const aio_proj* projs, int n_
 /*
  * The same, for a chained decoder step: projection i obtains its x as preps[i] says (AIO_X_*),
  * from buffers the caller filled or earlier projections of the step wrote; preps may be NULL (all
- * AIO_X_GIVEN).  projs[i].x receives the computed x.  A chained step takes M <= 4, and a computed x
- * is staged in shared memory, so M * (K + 32) * 2 must not exceed the staging area (35,360 bytes in
- * the default build: M = 1 for K = 11008, M <= 4 for K = 4096): UNSUPPORTED otherwise.  src, h_in, h_out and gamma must be
- * 16-byte aligned, src_stride and src_off multiples of 4: ALIGNMENT otherwise.  A missing pointer,
- * a column range outside src_stride, h_out == h_in or a negative eps: INVALID_ARG.  Device errors
- * are reported as for aio_decode_step_create.
+ * AIO_X_GIVEN).  projs[i].x receives the computed x.  A chained step takes M <= 4.  Every CTA computes
+ * an RMSNORM or SLICE x itself into shared memory, so M * (K + 32) * 2 must not exceed the staging
+ * area (35,360 bytes in the default build: M <= 4 for K = 4096): UNSUPPORTED otherwise.  A SWIGLU x
+ * that does not fit (M >= 2 at K = 5632 or 11008) is computed by a grid-wide phase of its own into
+ * projs[i].x instead (one more grid-wide step).  src, h_in, h_out and gamma must be 16-byte aligned,
+ * src_stride and src_off multiples of 4: ALIGNMENT otherwise.  A missing pointer, a column range
+ * outside src_stride, h_out == h_in or a negative eps: INVALID_ARG.  ATTENTION preparations: see
+ * aio_xprep.  Device errors are reported as for aio_decode_step_create.
  */
 aio_status aio_decode_step_create_chained(aio_step_t* out, const aio_proj* projs, const aio_xprep* preps,
                                           int n_projs, int M, unsigned flags);

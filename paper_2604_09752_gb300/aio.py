@@ -42,11 +42,12 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
-AIO_ABI_VERSION = 6
+AIO_ABI_VERSION = 7
 AIO_X_GIVEN = 0
 AIO_X_RMSNORM = 1
 AIO_X_SWIGLU = 2
 AIO_X_SLICE = 3
+AIO_X_ATTENTION = 4
 for _name, _val in re.findall(r"#define\s+(AIO_\w+)\s+(0x[0-9a-fA-F]+|\d+)u?\b", _hdr):
     if _name in globals() and globals()[_name] != int(_val, 0):
         raise ImportError(f"binding constant {_name} disagrees with include/aio.h")
@@ -68,7 +69,8 @@ class aio_proj(ctypes.Structure):
 class aio_xprep(ctypes.Structure):
     _fields_ = [("op", ctypes.c_int), ("src", ctypes.c_void_p), ("src_stride", ctypes.c_int),
                 ("src_off", ctypes.c_int), ("h_in", ctypes.c_void_p), ("h_out", ctypes.c_void_p),
-                ("gamma", ctypes.c_void_p), ("eps", ctypes.c_float)]
+                ("gamma", ctypes.c_void_p), ("eps", ctypes.c_float), ("kv_cache", ctypes.c_void_p),
+                ("L_past", ctypes.c_void_p), ("n_heads", ctypes.c_int), ("L_max", ctypes.c_int)]
 
 
 _vp, _int, _u = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint
@@ -194,7 +196,8 @@ def aio_decode_step_create(projs, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP
 
 def aio_decode_step_create_chained(projs, preps, M: int, flags: int = AIO_STEP_GRAPH | AIO_STEP_PERSISTENT) -> int:
     """projs as for aio_decode_step_create; preps: one (op, src, src_stride, src_off, h_in, h_out,
-    gamma, eps) tuple per projection, addresses as integers or None."""
+    gamma, eps[, kv_cache, L_past, n_heads, L_max]) tuple per projection, addresses as integers or
+    None."""
     assert len(preps) == len(projs)
     arr = (aio_proj * len(projs))(*[aio_proj(*p) for p in projs])
     parr = (aio_xprep * len(preps))(*[aio_xprep(*x) for x in preps])

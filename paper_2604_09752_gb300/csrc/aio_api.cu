@@ -120,6 +120,7 @@ struct aio_step {
     unsigned flags;
     bool persistent;
     bool chained;                        // some projection computes its x (the chained kernels run)
+    bool phases;                         // attention, merge or SwiGLU phases (their kernel instances)
     bool i8;                             // weight type of every projection (persistent mode)
     int grid;
     std::vector<aio::StreamArgs> chain;  // per-projection launches (chain mode)
@@ -405,12 +406,12 @@ static void step_free(aio_step* s) {
 
 static aio_status step_launch_all(aio_step* s, cudaStream_t stream) {
     if (s->persistent) {
-        AIO_CUDA(aio::launch_stream(s->whole, s->i8, s->grid, stream, false, true, s->chained));
+        AIO_CUDA(aio::launch_stream(s->whole, s->i8, s->grid, stream, false, true, s->chained, s->phases));
         return AIO_OK;
     }
     for (int i = 0; i < s->n; ++i) {
         const bool pdl = i > 0 && (s->flags & AIO_STEP_PDL);
-        AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false, s->chained));
+        AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false, s->chained, s->phases));
     }
     return AIO_OK;
 }
@@ -420,10 +421,26 @@ static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 // Host checks of one projection's x preparation (see aio_decode_step_create_chained).
 static aio_status validate_prep(const aio_linear* h, const aio_xprep& x, int M) {
     if (x.op == AIO_X_GIVEN) return AIO_OK;
+    const int K = h->K;
+    if (x.op == AIO_X_ATTENTION) {
+        // x is written by the step's merge phase and then staged like a given x
+        if (!x.src || !x.kv_cache || !x.L_past) return fail(AIO_ERR_INVALID_ARG, "ATTENTION needs src, kv_cache and L_past");
+        if (x.n_heads < 1 || static_cast<long long>(x.n_heads) * aio::kHeadDim != K)
+            return fail(AIO_ERR_INVALID_ARG, "ATTENTION needs K = 128 n_heads (K=%d, n_heads=%d)", K, x.n_heads);
+        if (x.n_heads > h->geo.Z) return fail(AIO_ERR_UNSUPPORTED, "n_heads=%d above the %d warps of the grid", x.n_heads, h->geo.Z);
+        if (x.L_max < M || static_cast<long long>(x.n_heads) * ((x.L_max + aio::kAttnPos - 1) / aio::kAttnPos) > (1LL << 30))
+            return fail(AIO_ERR_INVALID_ARG, "ATTENTION needs M <= L_max and n_heads * L_max / 16 <= 2^30 (L_max=%d)", x.L_max);
+        if (x.src_stride < 3LL * K) return fail(AIO_ERR_INVALID_ARG, "src_stride %d < 3K (%d)", x.src_stride, 3 * K);
+        if (!aligned16(x.src) || !aligned16(x.kv_cache) || !aligned(x.L_past, 4) || x.src_stride % 4 != 0)
+            return fail(AIO_ERR_ALIGNMENT, "src and kv_cache must be 16-byte aligned, L_past 4-byte, src_stride a multiple of 4");
+        if (aio::attn_merge_scratch(h->geo.Z) > aio::kXsBytes)
+            return fail(AIO_ERR_UNSUPPORTED, "a grid of %d warps: the attention merge lists do not fit", h->geo.Z);
+        return AIO_OK;
+    }
     if (x.op != AIO_X_RMSNORM && x.op != AIO_X_SWIGLU && x.op != AIO_X_SLICE)
         return fail(AIO_ERR_INVALID_ARG, "unknown x preparation %d", x.op);
-    const int K = h->K;
-    if (static_cast<long long>(M) * (K + aio::kXsPad) * 2 > aio::kXsBytes)
+    // a SwiGLU x that does not fit is computed by a grid-wide phase instead (see step_create)
+    if (x.op != AIO_X_SWIGLU && static_cast<long long>(M) * (K + aio::kXsPad) * 2 > aio::kXsBytes)
         return fail(AIO_ERR_UNSUPPORTED, "a computed x needs M (K + 32) 2 <= %d bytes (M=%d, K=%d)", aio::kXsBytes, M, K);
     if (x.op == AIO_X_RMSNORM) {
         if (!x.h_in || !x.gamma) return fail(AIO_ERR_INVALID_ARG, "RMSNORM needs h_in and gamma");
@@ -443,7 +460,13 @@ static aio_status validate_prep(const aio_linear* h, const aio_xprep& x, int M) 
     return AIO_OK;
 }
 
-static void apply_prep(aio::ProjDesc& d, const aio_xprep& x) {
+// A SwiGLU x too large for the staging area: computed into the projection's x by its own phase.
+static bool swiglu_phase(const aio_linear* h, const aio_xprep& x, int M) {
+    return x.op == AIO_X_SWIGLU && static_cast<long long>(M) * (h->K + aio::kXsPad) * 2 > aio::kXsBytes;
+}
+
+static void apply_prep(aio::ProjDesc& d, const aio_xprep& x, bool own_phase) {
+    if (x.op == AIO_X_ATTENTION || own_phase) return;   // an earlier phase writes x: staged (or read) as given
     d.xop = x.op;
     d.xsrc = x.src;
     d.xsrc_stride = x.op == AIO_X_RMSNORM ? d.K : x.src_stride;
@@ -492,27 +515,41 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
     for (int i = 0; preps && i < n_projs; ++i) chained = chained || preps[i].op != AIO_X_GIVEN;
     if (chained && M > aio::kMaxChainM)
         return fail(AIO_ERR_UNSUPPORTED, "a chained step supports M <= %d (M=%d)", aio::kMaxChainM, M);
+    bool phases = false;
+    for (int i = 0; preps && i < n_projs; ++i)
+        phases = phases || preps[i].op == AIO_X_ATTENTION || swiglu_phase(projs[i].h, preps[i], M);
     if (persistent) {
         int blocks = 0;
-        AIO_CUDA(aio::occupancy(wt0 == AIO_W_INT8_PERCHANNEL, M, chained, &blocks));
+        AIO_CUDA(aio::occupancy(wt0 == AIO_W_INT8_PERCHANNEL, M, chained, phases, &blocks));
         if (blocks < 1) return fail(AIO_ERR_UNSUPPORTED, "the stream kernel cannot be resident on an SM");
     }
+    // Phases: every projection, and before a projection whose x is attention over a KV cache, the
+    // attention phase and its merge.
+    int n_attn = 0, n_swiglu = 0;
+    for (int i = 0; preps && i < n_projs; ++i) {
+        n_attn += preps[i].op == AIO_X_ATTENTION ? 1 : 0;
+        n_swiglu += swiglu_phase(projs[i].h, preps[i], M) ? 1 : 0;
+    }
+    const int n_phases = n_projs + 2 * n_attn + n_swiglu;
+    const size_t apart_off = total;   // the attention phases' partial records (shared by the layers)
+    if (n_attn) total += round_up(static_cast<size_t>(projs[0].h->geo.Z) * 2 * M * aio::kAttnRec * sizeof(float), 256);
     const size_t desc_off = total;
-    total += round_up(sizeof(aio::ProjDesc) * n_projs, 256);
+    total += round_up(sizeof(aio::ProjDesc) * n_phases, 256);
     const size_t done_off = total;
-    total += round_up(sizeof(unsigned) * (n_projs + 1), 256);
+    total += round_up(sizeof(unsigned) * (n_phases + 1), 256);
     const size_t err_off = total;
-    total += round_up(sizeof(int) * n_projs, 256);
+    total += round_up(sizeof(int) * n_phases, 256);
     if (test_alloc_failure()) return fail(AIO_ERR_OOM, "workspace allocation failed (AIO_TEST_FAIL_ALLOC)");
     aio_step* s = new (std::nothrow) aio_step();
     if (!s) return fail(AIO_ERR_OOM, "host allocation failed");
     s->magic = kStepMagic;
     s->device = dev;
     s->M = M;
-    s->n = n_projs;
+    s->n = n_phases;
     s->flags = flags;
     s->persistent = persistent;
     s->chained = chained;
+    s->phases = phases;
     s->i8 = wt0 == AIO_W_INT8_PERCHANNEL;
     s->grid = grid;
     s->ws_bytes = total;
@@ -527,17 +564,79 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
     std::vector<aio::ProjDesc> descs;
     for (int i = 0; i < n_projs; ++i) {
         const aio_proj& p = projs[i];
+        const bool i8 = p.h->wt == AIO_W_INT8_PERCHANNEL;
+        if (preps && preps[i].op == AIO_X_ATTENTION) {
+            const aio_xprep& x = preps[i];
+            aio::ProjDesc a = {};
+            a.kind = aio::kPhaseAttn;
+            a.x = static_cast<const uint16_t*>(p.x);
+            a.K = a.N = p.h->K;
+            a.NG = a.NKT = 1;
+            a.xsrc = x.src;
+            a.xsrc_stride = x.src_stride;
+            a.kv = static_cast<uint16_t*>(x.kv_cache);
+            a.Lpast = x.L_past;
+            a.n_heads = x.n_heads;
+            a.L_max = x.L_max;
+            a.apart = reinterpret_cast<float*>(base + apart_off);
+            a.aout = static_cast<uint16_t*>(const_cast<void*>(p.x));
+            for (int kind : {aio::kPhaseAttn, aio::kPhaseMerge}) {
+                a.kind = kind;
+                descs.push_back(a);
+                const int e = static_cast<int>(descs.size()) - 1;
+                s->chain.push_back(aio::StreamArgs{});
+                s->chain.back() = single_args(p.h, a, M, s->errs + e);
+                s->chain_i8.push_back(i8 ? 1 : 0);
+            }
+        }
+        const bool own = preps && swiglu_phase(p.h, preps[i], M);
+        if (own) {
+            aio::ProjDesc g = {};
+            g.kind = aio::kPhaseSwiGlu;
+            g.x = static_cast<const uint16_t*>(p.x);
+            g.K = g.N = p.h->K;
+            g.NG = g.NKT = 1;
+            g.xsrc = preps[i].src;
+            g.xsrc_stride = preps[i].src_stride;
+            g.aout = static_cast<uint16_t*>(const_cast<void*>(p.x));
+            descs.push_back(g);
+            s->chain.push_back(single_args(p.h, g, M, s->errs + (descs.size() - 1)));
+            s->chain_i8.push_back(i8 ? 1 : 0);
+        }
         descs.push_back(make_desc(p.h, p.x, p.W, p.scales, p.y, reinterpret_cast<float*>(base + offs[i])));
-        if (preps) apply_prep(descs.back(), preps[i]);
-        s->chain.push_back(single_args(p.h, descs.back(), M, s->errs + i));
-        s->chain_i8.push_back(p.h->wt == AIO_W_INT8_PERCHANNEL ? 1 : 0);
+        if (preps) apply_prep(descs.back(), preps[i], own);
+        s->chain.push_back(single_args(p.h, descs.back(), M, s->errs + (descs.size() - 1)));
+        s->chain_i8.push_back(i8 ? 1 : 0);
+    }
+    // A projection whose x overlaps a buffer an earlier phase of the step writes (y, a computed x, a
+    // residual stream, an attention or SwiGLU output, a KV cache) reads data written in the same
+    // launch: it fences before staging x (generic stores, then async-proxy reads).
+    {
+        std::vector<std::pair<uintptr_t, uintptr_t>> written;
+        auto add = [&](const void* p, size_t n) {
+            if (p && n) written.emplace_back(reinterpret_cast<uintptr_t>(p), reinterpret_cast<uintptr_t>(p) + n);
+        };
+        for (aio::ProjDesc& d : descs) {
+            const size_t xb = static_cast<size_t>(M) * d.K * 2;
+            if (d.kind == aio::kPhaseProj) {
+                const uintptr_t a = reinterpret_cast<uintptr_t>(d.x);
+                for (const auto& r : written) d.xfence |= (a < r.second && r.first < a + xb) ? 1 : 0;
+                add(d.y, static_cast<size_t>(M) * d.N * 4);
+                if (d.xop != aio::kXGiven) add(d.x, xb);
+                add(d.h_out, static_cast<size_t>(M) * d.K * 4);
+            } else if (d.kind == aio::kPhaseAttn) {
+                add(d.kv, static_cast<size_t>(2) * d.n_heads * d.L_max * aio::kHeadDim * 2);
+            } else {
+                add(d.aout, xb);
+            }
+        }
     }
     aio::StreamArgs w = {};
     w.projs = reinterpret_cast<const aio::ProjDesc*>(base + desc_off);
     w.done = reinterpret_cast<unsigned*>(base + done_off);
-    w.exit_count = w.done + n_projs;
+    w.exit_count = w.done + n_phases;
     w.err = s->errs;
-    w.nproj = n_projs;
+    w.nproj = n_phases;
     w.M = M;
     w.Z = projs[0].h->geo.Z;
     w.test_stall = 0;
@@ -545,7 +644,7 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
     s->whole = w;
     if (cudaMemset(s->ws, 0xFF, desc_off) != cudaSuccess ||
         cudaMemset(base + desc_off, 0, total - desc_off) != cudaSuccess ||
-        cudaMemcpy(base + desc_off, descs.data(), sizeof(aio::ProjDesc) * n_projs, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(base + desc_off, descs.data(), sizeof(aio::ProjDesc) * n_phases, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaDeviceSynchronize() != cudaSuccess) {
         step_free(s);
         return fail(AIO_ERR_CUDA, "step workspace initialisation failed");

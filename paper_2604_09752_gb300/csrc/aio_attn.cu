@@ -23,13 +23,10 @@
 namespace aio {
 namespace {
 
-constexpr int kHeadDim = 128;
-constexpr int kAttnPos = 16;                                  // positions per unit
-constexpr int kAttnUnitBytes = kAttnPos * kHeadDim * 2;       // 4 KB of K (and of V) per unit
-constexpr int kAttnSlot = 2 * kAttnUnitBytes;                 // K then V
+// kHeadDim, kAttnPos (positions per unit), kAttnUnitBytes, kAttnSlot and kAttnRec (floats per
+// partial: 128 weighted V, max, sum, pad) are shared with the chained step (aio_internal.h).
 constexpr int kAttnStages = kRingBytesPerWarp / kAttnSlot;    // 3 slots of 8 KB per warp
 constexpr int kAttnSmem = kWarps * kAttnStages * kAttnSlot + kWarps * kAttnStages * 8;
-constexpr int kAttnRec = 132;                                 // floats per partial: 128 weighted V, max, sum, pad
 static_assert(kAttnStages >= 2, "attention ring");
 
 struct AttnArgs {
@@ -45,30 +42,6 @@ struct AttnArgs {
 };
 
 __device__ __forceinline__ long long attn_seg(long long z, long long U, int Z) { return z * U / Z; }
-
-__device__ __forceinline__ uint2 lds64(uint32_t addr) {
-    uint2 v;
-    asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
-    return v;
-}
-
-// Sum over the warp of 16 per-lane values a[0..15] (one per position); returns, in lane l, the
-// total for position (l >> 1) & 15.  Each step halves the values a lane holds: lanes whose bit o is
-// set keep the upper half and send the lower, the others the reverse, so 8 + 4 + 2 + 1 + 1 shuffles
-// replace 16 separate 5-step butterflies.
-__device__ __forceinline__ float warp_sum16_transpose(float (&a)[16], int lane) {
-#pragma unroll
-    for (int o = 16, n = 8; o >= 2; o >>= 1, n >>= 1) {
-        const bool hi = (lane & o) != 0;
-#pragma unroll
-        for (int i = 0; i < n; ++i) {
-            const float send = hi ? a[i] : a[i + n];
-            const float keep = hi ? a[i + n] : a[i];
-            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-    }
-    return a[0] + __shfl_xor_sync(0xffffffffu, a[0], 1);
-}
 
 template <int MT>
 __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __grid_constant__ AttnArgs a) {
@@ -158,70 +131,8 @@ __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __g
             dead = true;   // cslot is the slot that timed out; in_flight counts it
             break;
         }
-        {
-            // K and V rows are read from shared memory once for all tokens, and each step of the
-            // softmax runs for every token before the next, so the tokens' chains interleave.
-            const int p0 = c * kAttnPos, np = min(kAttnPos, a.L - p0);
-            const uint32_t kaddr = smem_addr(ring + cslot * kAttnSlot) + 8 * lane;
-            const uint32_t vaddr = kaddr + kAttnUnitBytes;
-            uint2 kr[kAttnPos], vr[kAttnPos];
-#pragma unroll
-            for (int j = 0; j < kAttnPos; ++j) {
-                kr[j] = j < np ? lds64(kaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
-                vr[j] = j < np ? lds64(vaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
-            }
-            // lanes 2p and 2p + 1 hold position p's score (base-2 logits)
-            const int pos = (lane >> 1) & 15;
-            float sc[MT], bm[MT];
-            bool vis[MT];
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                float part[kAttnPos];
-#pragma unroll
-                for (int j = 0; j < kAttnPos; ++j) {
-                    const float k0 = __uint_as_float(kr[j].x << 16), k1 = __uint_as_float(kr[j].x & 0xFFFF0000u);
-                    const float k2 = __uint_as_float(kr[j].y << 16), k3 = __uint_as_float(kr[j].y & 0xFFFF0000u);
-                    part[j] = fmaf(q4[m].w, k3, fmaf(q4[m].z, k2, fmaf(q4[m].y, k1, q4[m].x * k0)));
-                }
-                const float sm = warp_sum16_transpose(part, lane);
-                vis[m] = pos < np && p0 + pos <= a.L - a.M + m;
-                sc[m] = vis[m] ? sm : -INFINITY;
-                bm[m] = sc[m];
-            }
-#pragma unroll
-            for (int o = 2; o < 32; o <<= 1)
-#pragma unroll
-                for (int m = 0; m < MT; ++m) bm[m] = fmaxf(bm[m], __shfl_xor_sync(0xffffffffu, bm[m], o));
-            float pr[MT], ps[MT];
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                const float nm = fmaxf(mx[m], bm[m]);
-                const bool live = nm != -INFINITY;   // some position seen so far is visible
-                const float alpha = live ? exp2f(mx[m] - nm) : 1.0f;   // 0 while mx is -inf
-                pr[m] = live && vis[m] ? exp2f(sc[m] - nm) : 0.0f;
-                ps[m] = pr[m];
-                ls[m] *= alpha;
-                acc[m] = make_float4(acc[m].x * alpha, acc[m].y * alpha, acc[m].z * alpha, acc[m].w * alpha);
-                if (live) mx[m] = nm;
-            }
-#pragma unroll
-            for (int o = 2; o < 32; o <<= 1)
-#pragma unroll
-                for (int m = 0; m < MT; ++m) ps[m] += __shfl_xor_sync(0xffffffffu, ps[m], o);
-#pragma unroll
-            for (int m = 0; m < MT; ++m) ls[m] += ps[m];
-#pragma unroll
-            for (int j = 0; j < kAttnPos; ++j) {
-                const float v0 = __uint_as_float(vr[j].x << 16), v1 = __uint_as_float(vr[j].x & 0xFFFF0000u);
-                const float v2 = __uint_as_float(vr[j].y << 16), v3 = __uint_as_float(vr[j].y & 0xFFFF0000u);
-#pragma unroll
-                for (int m = 0; m < MT; ++m) {
-                    const float pj = __shfl_sync(0xffffffffu, pr[m], 2 * j);   // 0 past np: V is zero there too
-                    acc[m] = make_float4(fmaf(pj, v0, acc[m].x), fmaf(pj, v1, acc[m].y), fmaf(pj, v2, acc[m].z),
-                                         fmaf(pj, v3, acc[m].w));
-                }
-            }
-        }
+        attn_unit<MT>(smem_addr(ring + cslot * kAttnSlot) + 8 * lane, c * kAttnPos, min(kAttnPos, a.L - c * kAttnPos),
+                      a.L - a.M, q4, mx, ls, acc, lane);
         __syncwarp();   // every lane's reads of the slot are done before it is refilled
         const int done_slot = cslot;
         cslot = (cslot + 1 == kAttnStages) ? 0 : cslot + 1;

@@ -4,7 +4,8 @@
 
 namespace aio {
 
-StreamFn chain_stream_fn(bool i8, int M) {
+StreamFn chain_stream_fn(bool i8, int M, bool phases) {
+    if (phases) return chain_phase_stream_fn(i8, M);
     switch (M) {
         case 1: return i8 ? aio_stream_kernel<1, true, true> : aio_stream_kernel<1, false, true>;
         case 2: return i8 ? aio_stream_kernel<2, true, true> : aio_stream_kernel<2, false, true>;

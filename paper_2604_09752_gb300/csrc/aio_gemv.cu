@@ -81,18 +81,18 @@ StreamFn stream_fn(int M) {
     }
 }
 
-StreamFn kernel_for(bool i8, int M, bool chained) {
-    if (chained) return chain_stream_fn(i8, M);
+StreamFn kernel_for(bool i8, int M, bool chained, bool phases) {
+    if (chained) return chain_stream_fn(i8, M, phases);
     return i8 ? stream_fn<true>(M) : stream_fn<false>(M);
 }
 
 }  // namespace
 
 cudaError_t prepare_kernels() {
-    for (int ch = 0; ch < 2; ++ch) {
+    for (int ch = 0; ch < 3; ++ch) {   // plain, chained, chained with phases
         for (int i8 = 0; i8 < 2; ++i8) {
             for (int M = 1; M <= (ch ? kMaxChainM : kMaxM); ++M) {
-                StreamFn f = kernel_for(i8 != 0, M, ch != 0);
+                StreamFn f = kernel_for(i8 != 0, M, ch != 0, ch == 2);
                 cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
                 if (e != cudaSuccess) return e;
             }
@@ -101,8 +101,9 @@ cudaError_t prepare_kernels() {
     return cudaFuncSetAttribute(aio_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
 }
 
-cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop, bool chained) {
-    StreamFn f = kernel_for(i8, a.M, chained);
+cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop, bool chained,
+                          bool phases) {
+    StreamFn f = kernel_for(i8, a.M, chained, phases);
     if (!f) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(grid));
@@ -126,8 +127,8 @@ cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s
     return cudaLaunchKernelEx(&cfg, f, a);
 }
 
-cudaError_t occupancy(bool i8, int M, bool chained, int* blocks_per_sm) {
-    StreamFn f = kernel_for(i8, M, chained);
+cudaError_t occupancy(bool i8, int M, bool chained, bool phases, int* blocks_per_sm) {
+    StreamFn f = kernel_for(i8, M, chained, phases);
     if (!f) return cudaErrorInvalidValue;
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks_per_sm, f, kThreads, kSmemBytes);
 }

@@ -91,9 +91,29 @@ constexpr int kXsBytes = NarrowLayout::kXsBytes;
 constexpr int kDevErrTimeout = 1;       // a bulk-copy wait expired
 constexpr int kDevErrGridTimeout = 2;   // a wait for the previous projection expired
 constexpr int kDevErrPrep = 3;          // x preparation asked for a projection whose x is not staged
+constexpr int kDevErrAttn = 4;          // a chained step's attention: L_past + M outside [M, L_max]
 
 // How a projection's x is obtained (the values of AIO_X_*).
-constexpr int kXGiven = 0, kXRmsNorm = 1, kXSwiGlu = 2, kXSlice = 3;
+constexpr int kXGiven = 0, kXRmsNorm = 1, kXSwiGlu = 2, kXSlice = 3, kXAttention = 4;
+
+// Phases of a launch: a projection, or one of the two phases that compute an O projection's x by
+// attention over a KV cache in a chained step (the partial results of every warp's units, then
+// their merge).
+constexpr int kPhaseProj = 0, kPhaseAttn = 1, kPhaseMerge = 2;
+// ...or a phase that computes a projection's SwiGLU x into global memory, spread over the grid, when
+// it does not fit the staging area (the projection then reads it as a given x).
+constexpr int kPhaseSwiGlu = 3;
+
+// Decode attention: heads of 128, units of 16 positions of one head (4 KB of K and 4 KB of V, one
+// 8 KB ring slot), partial records of 128 weighted-V sums, the running max, the sum and padding.
+constexpr int kHeadDim = 128;
+constexpr int kAttnPos = 16;
+constexpr int kAttnUnitBytes = kAttnPos * kHeadDim * 2;
+constexpr int kAttnSlot = 2 * kAttnUnitBytes;
+constexpr int kAttnRec = 132;
+// Shared scratch of a chained step's attention merge for a grid of Z warps (it borrows the staged-x
+// area): the covering warps' record offsets and maxima, then each warp's partial sums.
+constexpr int attn_merge_scratch(int Z) { return (8 * Z + 15) / 16 * 16 + kWarps * 32 * 16 + kWarps * 4; }
 
 // One projection of a launch; read-only while the kernel runs.  Geometry:
 //   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles;
@@ -119,6 +139,16 @@ struct ProjDesc {
     int xsrc_stride;          // elements per token row of xsrc
     int xsrc_off;             // slice: first column
     float eps;                // RMSNorm
+    // Attention phases (kind kPhaseAttn / kPhaseMerge) before an O projection: q, k and v of the M
+    // new tokens are the column thirds of the QKV output xsrc (xsrc_stride elements per row, head h
+    // at columns [128 h, 128 h + 128) of each third).
+    uint16_t* kv;             // the layer's cache [2][n_heads][L_max][128] bf16, K then V
+    const int* Lpast;         // device int: positions in the cache before this step
+    float* apart;             // partial records [Z][2][M][kAttnRec]
+    uint16_t* aout;           // merge: the O projection's x [M][n_heads * 128] bf16; SwiGLU phase: x [M][K]
+    int kind;                 // kPhase*
+    int n_heads, L_max;
+    int xfence;               // 1: x may be written earlier in the same launch (fence before staging it)
 };
 static_assert(sizeof(ProjDesc) % 16 == 0, "descriptor array stride");
 
@@ -154,10 +184,13 @@ cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared 
 using StreamFn = void (*)(const StreamArgs);
 constexpr int kMaxChainM = 4;   // token rows of a chained step (its kernels are instantiated for M <= 4)
 static_assert(kMaxChainM < AIO_WIDE_M, "the chained step's staging limit is the narrow layout's");
-StreamFn chain_stream_fn(bool i8, int M);   // aio_chain.cu
+StreamFn chain_stream_fn(bool i8, int M, bool phases);   // aio_chain.cu
+StreamFn chain_phase_stream_fn(bool i8, int M);          // aio_chain_ph.cu
+// chained: the chained kernels (x computed on the device); phases: with attention, merge or SwiGLU
+// phases.
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop,
-                          bool chained = false);
-cudaError_t occupancy(bool i8, int M, bool chained, int* blocks_per_sm);
+                          bool chained = false, bool phases = false);
+cudaError_t occupancy(bool i8, int M, bool chained, bool phases, int* blocks_per_sm);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
 cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s);
 

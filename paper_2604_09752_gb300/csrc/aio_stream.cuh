@@ -134,6 +134,10 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// Orders this thread's earlier generic-proxy accesses (and those it has observed) before its later
+// async-proxy accesses, in every state space.
+__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
+
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
@@ -225,15 +229,54 @@ __device__ __forceinline__ size_t tile_offset(int K, int N, int g, int kt) {
     return (static_cast<size_t>(g) * kRows * K + static_cast<size_t>(kt) * rows * kKT) * E;
 }
 
-// What the issuing lane needs of one projection, held in registers.
+// What the issuing lane needs of one phase, held in registers.  A projection: its packed weights,
+// shape and tile grid.  An attention phase of a chained step streams units of 16 positions of one
+// head instead (T = n_heads * nch units, unit u = head u / nch, positions 16 (u % nch) ...): w is
+// the layer's KV cache, K = L_max, N = L (the cached positions including the new tokens), NKT = nch,
+// uniform = n_heads, rowmajor = kIssueAttn.  Merge and SwiGLU phases stream nothing (T = 0).
 struct IssueProj {
     const uint8_t* w;
     int Tq, Tr;           // T = Tq * Z + Tr
     int K, N, NKT;
     int uniform, rowmajor;
 };
+constexpr int kIssueAttn = 2;   // IssueProj::rowmajor of an attention phase
 
-__device__ __forceinline__ IssueProj load_issue(const ProjDesc* d) {
+// Positions an attention phase covers, L = L_past + M, read from the device int the caller set
+// before the launch; 0 when the cache cannot hold them (the phase then streams and computes nothing
+// and reports kDevErrAttn).
+__device__ __forceinline__ int attn_len(const ProjDesc* d, int M) {
+    const int lp = __ldg(d->Lpast);
+    return (lp >= 0 && lp <= d->L_max - M) ? lp + M : 0;
+}
+
+// Units and segment bounds of an attention (or merge) phase over Z warps.
+__device__ __forceinline__ void attn_geom(const ProjDesc* d, int M, int Z, int& L, int& nch, int& Tq, int& Tr) {
+    L = attn_len(d, M);
+    nch = (L + kAttnPos - 1) / kAttnPos;
+    const int U = d->kind == kPhaseAttn ? d->n_heads * nch : 0;
+    Tq = U / Z;
+    Tr = U - Tq * Z;
+}
+
+// The issue fields of a chained step's non-projection phase (out of line: it runs once per phase).
+__device__ __noinline__ IssueProj load_issue_phase(const ProjDesc* d, int M, int Z) {
+    IssueProj q;
+    int L = 0, nch = 0;
+    q.Tq = q.Tr = 0;   // merge and SwiGLU phases stream nothing
+    if (d->kind == kPhaseAttn) attn_geom(d, M, Z, L, nch, q.Tq, q.Tr);
+    q.w = reinterpret_cast<const uint8_t*>(d->kv);
+    q.K = d->L_max;
+    q.N = L;
+    q.NKT = nch;
+    q.uniform = d->n_heads;
+    q.rowmajor = kIssueAttn;
+    return q;
+}
+
+template <bool PH>
+__device__ __forceinline__ IssueProj load_issue(const ProjDesc* d, int M, int Z) {
+    if (PH && d->kind != kPhaseProj) return load_issue_phase(d, M, Z);
     IssueProj q;
     q.w = d->w;
     q.Tq = d->Tq;
@@ -244,6 +287,19 @@ __device__ __forceinline__ IssueProj load_issue(const ProjDesc* d) {
     q.uniform = d->uniform;
     q.rowmajor = d->rowmajor;
     return q;
+}
+
+// Lane 0: the K rows then the V rows of attention unit u into one slot (K at dst, V at dst +
+// kAttnUnitBytes), both 256 B per position, completing on the slot's barrier.
+__device__ __noinline__ void issue_attn_unit(IssueProj d, int u, uint8_t* dst, uint64_t* bar, uint64_t pol) {
+    const int h = u / d.NKT, c = u - h * d.NKT;
+    const int p0 = c * kAttnPos, np = min(kAttnPos, d.N - p0);
+    const uint32_t bytes = static_cast<uint32_t>(np * kHeadDim * 2);
+    const size_t off = (static_cast<size_t>(h) * d.K + p0) * (kHeadDim * 2);
+    const size_t voff = static_cast<size_t>(d.uniform) * d.K * (kHeadDim * 2);
+    mbar_expect_tx(bar, 2 * bytes);
+    bulk_g2s(dst, d.w + off, bytes, bar, pol);
+    bulk_g2s(dst + kAttnUnitBytes, d.w + voff + off, bytes, bar, pol);
 }
 
 // First tile of warp z's segment (z = Z gives T): floor(z T / Z) = z Tq + floor(z Tr / Z), exact in
@@ -314,28 +370,31 @@ struct ChunkCursor {
     IssueProj cur, nxt;
 };
 
+template <bool PH>
 __device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, int z, int Z) {
-    c.cur = load_issue(proj_desc(s, 0));
-    c.nxt = s.nproj > 1 ? load_issue(proj_desc(s, 1)) : c.cur;
+    c.cur = load_issue<PH>(proj_desc(s, 0), s.M, Z);
+    c.nxt = s.nproj > 1 ? load_issue<PH>(proj_desc(s, 1), s.M, Z) : c.cur;
     c.p = 0;
     c.t = seg(z, Z, c.cur.Tq, c.cur.Tr);
     c.te = seg(z + 1, Z, c.cur.Tq, c.cur.Tr);
 }
 
-// Next chunk of the walk: its projection, first tile and tile count; false at the end.
+// Next chunk of the walk: its phase, first tile (or unit) and count; false at the end.  An
+// attention unit fills a slot on its own.
+template <bool PH>
 __device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s, int z, int Z, int C, int& p,
                                             int& t, int& nt) {
     while (c.t >= c.te) {
         if (c.p + 1 >= s.nproj) return false;
         ++c.p;
         c.cur = c.nxt;
-        if (c.p + 1 < s.nproj) c.nxt = load_issue(proj_desc(s, c.p + 1));
+        if (c.p + 1 < s.nproj) c.nxt = load_issue<PH>(proj_desc(s, c.p + 1), s.M, Z);
         c.t = seg(z, Z, c.cur.Tq, c.cur.Tr);
         c.te = seg(z + 1, Z, c.cur.Tq, c.cur.Tr);
     }
     p = c.p;
     t = c.t;
-    nt = min(C, c.te - c.t);
+    nt = (PH && c.cur.rowmajor == kIssueAttn) ? 1 : min(C, c.te - c.t);
     c.t += nt;
     return true;
 }
@@ -351,8 +410,10 @@ struct Proj {
     int M, K, N, NKT;
     int rowmajor, uniform;
     int xop;
+    int xfence;   // plain kernels: fence before staging x (chained kernels always fence)
 };
 
+template <bool CH>
 __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
     Proj p;
     p.x = d->x;
@@ -369,6 +430,7 @@ __device__ __forceinline__ Proj load_proj(const ProjDesc* d, int M) {
     p.rowmajor = d->rowmajor;
     p.uniform = d->uniform;
     p.xop = d->xop;
+    p.xfence = CH ? 1 : d->xfence;
     return p;
 }
 
@@ -516,10 +578,11 @@ __device__ __forceinline__ void ffma_full_g(float (&d)[4][4], const uint8_t* til
 // (rows < 16 or klen < 256) and row-major weights as the row-major block [rows][klen].  Pieces
 // outside the tile are zero, and so is x outside [kbase, kbase + klen) or for tokens >= M.
 // x is read from xp = x + token g's row (row stride xstride elements), staged or global.
+// x_l2: xrow_ptr is global memory other CTAs may have written earlier in the launch (read at L2).
 template <bool I8>
 __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, int rows, int klen, int kbase,
                                          int lane, const Proj& P, const uint16_t* xrow_ptr, const I8Consts& kc,
-                                         int xstride = 0) {
+                                         int xstride = 0, bool x_l2 = false) {
     using TL = TileT<I8>;
     constexpr int NP = TL::kPieces;
     const int g = lane >> 2, c = lane & 3;
@@ -563,7 +626,8 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
 #pragma unroll
     for (int t = 0; t < kRuns; ++t) {
         const int k = 32 * t + 8 * c;
-        xv[t] = (xrow && k < klen) ? *reinterpret_cast<const uint4*>(xrow_ptr + kbase + k) : make_uint4(0u, 0u, 0u, 0u);
+        const uint4* xq = reinterpret_cast<const uint4*>(xrow_ptr + kbase + k);
+        xv[t] = (xrow && k < klen) ? (x_l2 ? __ldcg(xq) : *xq) : make_uint4(0u, 0u, 0u, 0u);
     }
     tile_mma_frag<I8>(d, w, xv, kc);
 #endif
@@ -572,7 +636,9 @@ __device__ __forceinline__ void tile_mma(float (&d)[4][4], const uint8_t* tile, 
 // A full packed tile with x in global memory: xp = x + token min(g, M-1)'s row + 256 kt + 8c.
 // Lanes g >= M load a real token's x (the same addresses as lanes of token M-1, served once):
 // they only fill columns of D for tokens >= M, which are never written.  No select is needed.
-template <bool I8>
+// CG: x may have been written by other CTAs earlier in the launch (a chained step's SwiGLU phase),
+// so it is read at L2 rather than through L1.
+template <bool I8, bool CG = false>
 __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* tile_lane, const uint16_t* xp,
                                               const I8Consts& kc) {
     using TL = TileT<I8>;
@@ -581,7 +647,10 @@ __device__ __forceinline__ void tile_mma_full(float (&d)[4][4], const uint8_t* t
     for (int j = 0; j < TL::kPieces; ++j) w[j] = *reinterpret_cast<const uint4*>(tile_lane + j * 512);
     uint4 xv[kRuns];
 #pragma unroll
-    for (int t = 0; t < kRuns; ++t) xv[t] = *reinterpret_cast<const uint4*>(xp + 32 * t);
+    for (int t = 0; t < kRuns; ++t) {
+        const uint4* xq = reinterpret_cast<const uint4*>(xp + 32 * t);
+        xv[t] = CG ? __ldcg(xq) : *xq;
+    }
     tile_mma_frag<I8>(d, w, xv, kc);
 }
 
@@ -795,6 +864,115 @@ __device__ __forceinline__ unsigned cta_arrive(unsigned* cta_count, unsigned* gl
         }
     }
     return __shfl_sync(0xffffffffu, g, 0);
+}
+
+// ------------------------------------------------------------------ decode attention
+// Shared by the attention kernel (aio_attn.cu) and the attention phases of a chained step.
+__device__ __forceinline__ uint2 lds64(uint32_t addr) {
+    uint2 v;
+    asm volatile("ld.shared.v2.b32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+// Sum over the warp of 16 per-lane values a[0..15] (one per position); returns, in lane l, the
+// total for position (l >> 1) & 15.  Each step halves the values a lane holds: lanes whose bit o is
+// set keep the upper half and send the lower, the others the reverse, so 8 + 4 + 2 + 1 + 1 shuffles
+// replace 16 separate 5-step butterflies.
+__device__ __forceinline__ float warp_sum16_transpose(float (&a)[16], int lane) {
+#pragma unroll
+    for (int o = 16, n = 8; o >= 2; o >>= 1, n >>= 1) {
+        const bool hi = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < n; ++i) {
+            const float send = hi ? a[i] : a[i + n];
+            const float keep = hi ? a[i + n] : a[i];
+            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    return a[0] + __shfl_xor_sync(0xffffffffu, a[0], 1);
+}
+
+// One unit of np <= 16 positions [p0, p0 + np) of one head, staged in shared memory: K rows at
+// kaddr - 8 lane (256 B apart), V rows kAttnUnitBytes later.  Token m sits at position q0 + m and
+// sees positions j <= q0 + m.  Lane l holds dims [4l, 4l + 4) of each token's q (scaled by
+// log2(e) / sqrt(128)) and of its running weighted V sum; mx and ls are the running base-2 max and
+// sum of an online softmax.  K and V rows are read from shared memory once for all tokens, and
+// each step of the softmax runs for every token before the next, so the tokens' chains interleave.
+// PRELOAD: all 16 K and V rows are loaded first (more loads in flight, 64 more registers).
+template <int MT, bool PRELOAD = true>
+__device__ __forceinline__ void attn_unit(uint32_t kaddr, int p0, int np, int q0, const float4 (&q4)[MT],
+                                          float (&mx)[MT], float (&ls)[MT], float4 (&acc)[MT], int lane) {
+    const uint32_t vaddr = kaddr + kAttnUnitBytes;
+    constexpr int NR = PRELOAD ? kAttnPos : 1;
+    uint2 kr[NR], vr[NR];
+    auto krow = [&](int j) -> uint2 {
+        if constexpr (PRELOAD) return kr[j];
+        return j < np ? lds64(kaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+    };
+    auto vrow = [&](int j) -> uint2 {
+        if constexpr (PRELOAD) return vr[j];
+        return j < np ? lds64(vaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+    };
+    if constexpr (PRELOAD) {
+#pragma unroll
+        for (int j = 0; j < kAttnPos; ++j) {
+            kr[j] = j < np ? lds64(kaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+            vr[j] = j < np ? lds64(vaddr + j * (kHeadDim * 2)) : make_uint2(0u, 0u);
+        }
+    }
+    // lanes 2p and 2p + 1 hold position p's score (base-2 logits)
+    const int pos = (lane >> 1) & 15;
+    float sc[MT], bm[MT];
+    bool vis[MT];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+        float part[kAttnPos];
+#pragma unroll
+        for (int j = 0; j < kAttnPos; ++j) {
+            const uint2 kj = krow(j);
+            const float k0 = __uint_as_float(kj.x << 16), k1 = __uint_as_float(kj.x & 0xFFFF0000u);
+            const float k2 = __uint_as_float(kj.y << 16), k3 = __uint_as_float(kj.y & 0xFFFF0000u);
+            part[j] = fmaf(q4[m].w, k3, fmaf(q4[m].z, k2, fmaf(q4[m].y, k1, q4[m].x * k0)));
+        }
+        const float sm = warp_sum16_transpose(part, lane);
+        vis[m] = pos < np && p0 + pos <= q0 + m;
+        sc[m] = vis[m] ? sm : -INFINITY;
+        bm[m] = sc[m];
+    }
+#pragma unroll
+    for (int o = 2; o < 32; o <<= 1)
+#pragma unroll
+        for (int m = 0; m < MT; ++m) bm[m] = fmaxf(bm[m], __shfl_xor_sync(0xffffffffu, bm[m], o));
+    float pr[MT], ps[MT];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+        const float nm = fmaxf(mx[m], bm[m]);
+        const bool live = nm != -INFINITY;   // some position seen so far is visible
+        const float alpha = live ? exp2f(mx[m] - nm) : 1.0f;   // 0 while mx is -inf
+        pr[m] = live && vis[m] ? exp2f(sc[m] - nm) : 0.0f;
+        ps[m] = pr[m];
+        ls[m] *= alpha;
+        acc[m] = make_float4(acc[m].x * alpha, acc[m].y * alpha, acc[m].z * alpha, acc[m].w * alpha);
+        if (live) mx[m] = nm;
+    }
+#pragma unroll
+    for (int o = 2; o < 32; o <<= 1)
+#pragma unroll
+        for (int m = 0; m < MT; ++m) ps[m] += __shfl_xor_sync(0xffffffffu, ps[m], o);
+#pragma unroll
+    for (int m = 0; m < MT; ++m) ls[m] += ps[m];
+#pragma unroll
+    for (int j = 0; j < kAttnPos; ++j) {
+        const uint2 vj = vrow(j);
+        const float v0 = __uint_as_float(vj.x << 16), v1 = __uint_as_float(vj.x & 0xFFFF0000u);
+        const float v2 = __uint_as_float(vj.y << 16), v3 = __uint_as_float(vj.y & 0xFFFF0000u);
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            const float pj = __shfl_sync(0xffffffffu, pr[m], 2 * j);   // 0 past np: V is zero there too
+            acc[m] = make_float4(fmaf(pj, v0, acc[m].x), fmaf(pj, v1, acc[m].y), fmaf(pj, v2, acc[m].z),
+                                 fmaf(pj, v3, acc[m].w));
+        }
+    }
 }
 
 // ------------------------------------------------------------------ x of a chained step
@@ -1023,15 +1201,235 @@ __device__ __forceinline__ void prep_x(const ProjDesc* d, uint16_t* xs, int xs_s
     named_barrier_sync();
 }
 
+// The merge phase of a chained step's attention.  CTA c merges the (head, token) items c, c + G,
+// ...: the records of the warps whose units cover the head are listed in shared memory, each warp
+// adds records w, w + 8, ... weighted by 2^(max_r - max), and warp 0 adds the warps' results in
+// order (a fixed order, whatever the timing), divides by the total weight and writes the head's
+// slice of the O projection's x row as bf16.  Every warp of a CTA takes part (named barriers),
+// whatever its state.
+template <int MT>
+__device__ __noinline__ void attn_merge(const ProjDesc* d, int Z, uint8_t* scratch, int warp, int lane) {
+    const int L = attn_len(d, MT);
+    if (L == 0) return;
+    const int nch = (L + kAttnPos - 1) / kAttnPos;
+    const int U = d->n_heads * nch, Tq = U / Z, Tr = U - Tq * Z;
+    const int items = d->n_heads * MT, H = d->n_heads * kHeadDim;
+    int* srec = reinterpret_cast<int*>(scratch);
+    float* smx = reinterpret_cast<float*>(scratch + 4 * Z);
+    float4* wacc = reinterpret_cast<float4*>(scratch + (8 * Z + 15) / 16 * 16);
+    float* wl = reinterpret_cast<float*>(wacc + kWarps * 32);
+    const int tid = warp * 32 + lane;
+    for (int it = blockIdx.x; it < items; it += gridDim.x) {
+        const int h = it / MT, m = it - h * MT;
+        const int ua = h * nch, ub = ua + nch - 1;   // the head's units
+        // the warps holding units ua and ub (segment starts are nondecreasing in z)
+        int zlo = static_cast<int>(static_cast<long long>(ua) * Z / U);
+        while (zlo > 0 && seg(zlo, Z, Tq, Tr) > ua) --zlo;
+        while (seg(zlo + 1, Z, Tq, Tr) <= ua) ++zlo;
+        int zhi = static_cast<int>(static_cast<long long>(ub) * Z / U);
+        while (zhi > 0 && seg(zhi, Z, Tq, Tr) > ub) --zhi;
+        while (seg(zhi + 1, Z, Tq, Tr) <= ub) ++zhi;
+        const int n = zhi - zlo + 1;
+        for (int i = tid; i < n; i += kThreads) {
+            const int zz = zlo + i, s0 = seg(zz, Z, Tq, Tr);
+            int r = -1;
+            float mxv = -INFINITY;
+            if (seg(zz + 1, Z, Tq, Tr) > s0) {   // a non-empty segment: its first or second record
+                r = ((zz * 2 + (s0 / nch == h ? 0 : 1)) * MT + m) * kAttnRec;
+                mxv = __ldcg(d->apart + r + 128);
+            }
+            srec[i] = r;
+            smx[i] = mxv;
+        }
+        named_barrier_sync();
+        float gm = -INFINITY;
+        for (int i = lane; i < n; i += 32) gm = fmaxf(gm, smx[i]);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
+        float l = 0.0f;
+        float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll 4
+        for (int i = warp; i < n; i += kWarps) {
+            const int r = srec[i];
+            if (r < 0) continue;
+            const float w = smx[i] == -INFINITY ? 0.0f : exp2f(smx[i] - gm);
+            l = fmaf(__ldcg(d->apart + r + 129), w, l);
+            const float4 v = ldcg4(d->apart + r + 4 * lane);
+            a = make_float4(fmaf(v.x, w, a.x), fmaf(v.y, w, a.y), fmaf(v.z, w, a.z), fmaf(v.w, w, a.w));
+        }
+        wacc[warp * 32 + lane] = a;
+        if (lane == 0) wl[warp] = l;
+        named_barrier_sync();
+        if (warp == 0) {
+            float lt = 0.0f;
+            float4 at = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) {
+                lt += wl[w];
+                const float4 v = wacc[w * 32 + lane];
+                at = make_float4(at.x + v.x, at.y + v.y, at.z + v.z, at.w + v.w);
+            }
+            const float inv = 1.0f / lt;
+            *reinterpret_cast<uint2*>(d->aout + static_cast<size_t>(m) * H + h * kHeadDim + 4 * lane) =
+                make_uint2(bf16x2_rn(at.x * inv, at.y * inv), bf16x2_rn(at.z * inv, at.w * inv));
+        }
+        named_barrier_sync();   // the lists are read before the next item rewrites them
+    }
+    fence_proxy_async_smem();   // the scratch writes precede the next phase's bulk copies into this area
+}
+
+// A warp's ring state, handed to and returned by the out-of-line attention phase.
+struct RingCtx {
+    ChunkCursor cur;
+    int islot, in_flight, ahead, cslot;
+    uint32_t cphase;
+    bool first_issue, dead;
+};
+
+// The attention phase of a chained step, for one warp: attention of the M new tokens over the
+// layer's cache, over this warp's units, each one ring slot of 16 positions of one head.  The new
+// tokens' rows (positions L_past .. L - 1) were copied stale from the cache: they are replaced by k
+// and v of the QKV output rounded to bf16, which are also written back to the cache.  A warp's units
+// span at most two heads (n_heads <= Z), so it leaves at most two partial records.  The ring is
+// refilled as in the projection phases (the issue and refill steps of the stream kernel, restated
+// on the state passed in).
+template <int MT, bool I8>
+__device__ __noinline__ RingCtx attn_phase(RingCtx r, const StreamArgs& s, const ProjDesc* D, uint8_t* ring,
+                                           uint64_t* bars, int z, int lane, uint64_t pol, int p) {
+    using TL = TileT<I8>;
+    using SL = LayoutFor<MT>;
+    constexpr int C = TL::kChunk;
+    constexpr int S = I8 ? SL::kStagesI8 : SL::kStages;
+    const int Z = s.Z;
+    auto issue_next = [&]() -> bool {
+        int ip, it, nt;
+        if (!cursor_next<true>(r.cur, s, z, Z, C, ip, it, nt)) return false;
+        if (lane == 0) {
+            if (r.cur.cur.rowmajor == kIssueAttn)
+                issue_attn_unit(r.cur.cur, it, ring + r.islot * TL::kSlot, &bars[r.islot], pol);
+            else
+                issue_chunk<I8>(r.cur.cur, it, nt, ring + r.islot * TL::kSlot, &bars[r.islot], pol);
+        }
+        r.first_issue = false;
+        r.islot = (r.islot + 1 == S) ? 0 : r.islot + 1;
+        return true;
+    };
+    auto refill = [&]() {
+        const bool later = r.cur.p > p || r.cur.t >= r.cur.te;
+        if (later && r.ahead >= TL::kAheadLive) {
+            --r.in_flight;
+            return;
+        }
+        if (!issue_next()) {
+            --r.in_flight;
+        } else if (later) {
+            ++r.ahead;
+        }
+    };
+    int L, nch, Tq, Tr;
+    attn_geom(D, MT, Z, L, nch, Tq, Tr);
+    if (L == 0 && z == 0 && lane == 0) atomicCAS(s.err, 0, kDevErrAttn);
+    const int u0 = seg(z, Z, Tq, Tr), u1 = seg(z + 1, Z, Tq, Tr);
+    const int H = D->n_heads * kHeadDim, qs = D->xsrc_stride, Lp = L - MT;
+    const float* qkv = D->xsrc;
+    uint16_t* kvc = D->kv;
+    const size_t voff = static_cast<size_t>(D->n_heads) * D->L_max * kHeadDim;
+    const float qscale = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));   // log2(e) / sqrt(d)
+    float4 q4[MT], acc[MT];
+    float mx[MT], ls[MT];
+    int head = -1, sidx = -1;
+    auto flush = [&]() {
+        if (head < 0) return;
+        float* base = D->apart + (static_cast<size_t>(z) * 2 + sidx) * MT * kAttnRec;
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            float* rec = base + m * kAttnRec;
+            *reinterpret_cast<float4*>(rec + 4 * lane) = acc[m];
+            if (lane == 0) {
+                rec[128] = mx[m];
+                rec[129] = ls[m];
+            }
+        }
+    };
+    int h = nch ? u0 / nch : 0, c = u0 - h * nch - 1;
+    for (int u = u0; u < u1 && !r.dead; ++u) {
+        if (++c == nch) {
+            c = 0;
+            ++h;
+        }
+        if (h != head) {
+            flush();
+            head = h;
+            ++sidx;
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+                const float4 t = ldcg4(qkv + static_cast<size_t>(m) * qs + h * kHeadDim + 4 * lane);
+                q4[m] = make_float4(t.x * qscale, t.y * qscale, t.z * qscale, t.w * qscale);
+                mx[m] = -INFINITY;
+                ls[m] = 0.0f;
+                acc[m] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            }
+        }
+        if (!__all_sync(0xffffffffu, mbar_wait(&bars[r.cslot], r.cphase, s.wait_limit_ns))) {
+            if (lane == 0) atomicExch(s.err, kDevErrTimeout);
+            r.dead = true;
+            break;
+        }
+        const int p0 = c * kAttnPos, np = min(kAttnPos, L - p0);
+        uint8_t* slot = ring + r.cslot * TL::kSlot;
+        const int jn0 = max(p0, Lp), jn1 = p0 + np;
+        if (jn0 < jn1) {
+            for (int j = jn0; j < jn1; ++j) {
+                const int m = j - Lp, row = j - p0;
+                const float* src = qkv + static_cast<size_t>(m) * qs + h * kHeadDim + 4 * lane;
+                const float4 kf = ldcg4(src + H), vf = ldcg4(src + 2 * H);
+                const uint2 kb = make_uint2(bf16x2_rn(kf.x, kf.y), bf16x2_rn(kf.z, kf.w));
+                const uint2 vb = make_uint2(bf16x2_rn(vf.x, vf.y), bf16x2_rn(vf.z, vf.w));
+                *reinterpret_cast<uint2*>(slot + row * (kHeadDim * 2) + 8 * lane) = kb;
+                *reinterpret_cast<uint2*>(slot + kAttnUnitBytes + row * (kHeadDim * 2) + 8 * lane) = vb;
+                const size_t off = (static_cast<size_t>(h) * D->L_max + j) * kHeadDim + 4 * lane;
+                *reinterpret_cast<uint2*>(kvc + off) = kb;
+                *reinterpret_cast<uint2*>(kvc + voff + off) = vb;
+            }
+            fence_proxy_async_smem();   // these writes precede the slot's next bulk copy
+            __syncwarp();               // every lane's rows are in place before any lane reads
+        }
+        attn_unit<MT, false>(smem_addr(slot) + 8 * lane, p0, np, Lp, q4, mx, ls, acc, lane);
+        __syncwarp();   // every lane's reads of the slot are done before it is refilled
+        r.cslot = (r.cslot + 1 == S) ? 0 : r.cslot + 1;
+        r.cphase ^= (r.cslot == 0) ? 1u : 0u;
+        refill();
+    }
+    flush();
+    if (!r.dead) {
+        while (r.ahead < TL::kAhead && r.in_flight < S && issue_next()) {
+            ++r.in_flight;
+            ++r.ahead;
+        }
+    } else {
+        // wait (bounded) for this warp's copies still in flight, then stop issuing
+        for (int j = 0; j < r.in_flight; ++j) {
+            mbar_wait(&bars[r.cslot], r.cphase, s.wait_limit_ns);
+            r.cslot = (r.cslot + 1 == S) ? 0 : r.cslot + 1;
+            r.cphase ^= (r.cslot == 0) ? 1u : 0u;
+        }
+        r.in_flight = 0;
+    }
+    return r;
+}
+
 // The stream kernel: one CTA per SM, every warp streams its segment of every projection through
 // its own bulk-copy ring.  All per-tile bookkeeping is incremental 32-bit arithmetic; divisions
 // happen once per chunk (issue) or once per projection (consume).  CH: a chained step, where a
 // projection's x may be computed on the device (prep_x); the plain step's kernels carry none of
-// that code.
-template <int MT, bool I8, bool CH>
+// that code.  PH: a chained step that also has attention, merge or SwiGLU phases (their own
+// instantiations, so that the chained kernels without them keep their registers for the projections).
+template <int MT, bool I8, bool CH, bool PH = false>
 __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_constant__ StreamArgs s) {
     using TL = TileT<I8>;
     using SL = LayoutFor<MT>;
+    static_assert(CH || !PH, "phases belong to chained steps");
+    static_assert(!PH || TL::kSlot >= kAttnSlot, "a ring slot holds one attention unit");
     constexpr int C = TL::kChunk;
     constexpr int S = I8 ? SL::kStagesI8 : SL::kStages;   // ring slots per warp
     constexpr int E = TL::kEsize;
@@ -1069,15 +1467,18 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
 
     // The issue cursor walks this warp's tiles of all projections in consumption order.
     ChunkCursor ring_cur;
-    cursor_init(ring_cur, s, z, Z);
+    cursor_init<PH>(ring_cur, s, static_cast<int>(z), Z);
     int islot = 0;
     bool first_issue = true;
     const bool stall = s.test_stall && z == Z - 1;   // the grid's last warp always owns >= 1 tile
     auto issue_next = [&]() -> bool {
         int ip, it, nt;
-        if (!cursor_next(ring_cur, s, z, Z, C, ip, it, nt)) return false;
-        if (lane == 0 && !(stall && first_issue))   // test hook: this slot's barrier never completes
+        if (!cursor_next<PH>(ring_cur, s, static_cast<int>(z), Z, C, ip, it, nt)) return false;
+        if (PH && ring_cur.cur.rowmajor == kIssueAttn) {
+            if (lane == 0) issue_attn_unit(ring_cur.cur, it, ring + islot * TL::kSlot, &bars[islot], pol);
+        } else if (lane == 0 && !(stall && first_issue)) {   // test hook: this slot's barrier never completes
             issue_chunk<I8>(ring_cur.cur, it, nt, ring + islot * TL::kSlot, &bars[islot], pol);
+        }
         first_issue = false;
         islot = (islot + 1 == S) ? 0 : islot + 1;
         return true;
@@ -1114,17 +1515,23 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
     uint32_t xphase = 0;
     bool dead = false;    // set after a timeout: stop consuming, keep signalling
     for (int p = 0; p < s.nproj; ++p) {
-        Proj P = load_proj(proj_desc(s, p), MT);
+        Proj P = load_proj<CH>(proj_desc(s, p), MT);
+        // the phase kind is reloaded where it is needed (the chained kernels are short of registers)
+        auto kind_of = [&]() { return PH ? proj_desc(s, p)->kind : kPhaseProj; };
         const long long t0 = seg(static_cast<int>(z), Z, P.Tq, P.Tr), t1 = seg(static_cast<int>(z) + 1, Z, P.Tq, P.Tr);
         // Staged x rows are kXsPad elements apart beyond K, so two tokens read in one shared-memory
         // phase fall in different banks.
         const int xs_stride = P.K + kXsPad;
-        const bool stage = P.M * xs_stride * 2 <= SL::kXsBytes;
+        const bool stage = kind_of() == kPhaseProj && P.M * xs_stride * 2 <= SL::kXsBytes;
         // Warp 0 stages x once every CTA has finished the previous projection (every warp of this
         // CTA has then finished reading the previous x and fenced its reads against async writes):
-        // one bulk copy per token row.
+        // one bulk copy per token row.  When x may have been written by other CTAs earlier in the
+        // launch (generic stores, ordered before the grid counter's acquire), a proxy fence orders
+        // them before these async-proxy reads: in a chained step whenever x is staged as given (the
+        // O projection after attention), in a plain step where the host found x aliased.
         auto stage_x = [&]() {
             if (stage && (!CH || P.xop == kXGiven) && lane == 0) {
+                if (CH || P.xfence) fence_proxy_async_all();
                 mbar_expect_tx(xbar, static_cast<uint32_t>(P.M * P.K * 2));
                 for (int m = 0; m < P.M; ++m)
                     bulk_g2s_plain(xs + m * xs_stride, P.x + static_cast<size_t>(m) * P.K,
@@ -1177,7 +1584,35 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         if (!dead) {
             while (in_flight < S && issue_next()) ++in_flight;
         }
-        if (!dead && t1 > t0) {
+        if constexpr (PH) {
+            const int kind = kind_of();
+            if (kind == kPhaseAttn) {
+                RingCtx rc{ring_cur, islot, in_flight, ahead, cslot, cphase, first_issue, dead};
+                rc = attn_phase<MT, I8>(rc, s, proj_desc(s, p), ring, bars, static_cast<int>(z), lane, pol, p);
+                ring_cur = rc.cur;
+                islot = rc.islot;
+                in_flight = rc.in_flight;
+                ahead = rc.ahead;
+                cslot = rc.cslot;
+                cphase = rc.cphase;
+                first_issue = rc.first_issue;
+                dead = rc.dead;
+            } else if (kind == kPhaseMerge) {
+                attn_merge<MT>(proj_desc(s, p), Z, reinterpret_cast<uint8_t*>(xs), warp, lane);
+            } else if (kind == kPhaseSwiGlu) {
+                // x[m, k] = bf16(silu(src[m, k]) * src[m, K + k]), four values per thread, over the grid
+                const ProjDesc* D = proj_desc(s, p);
+                const int K = D->K, n4 = K / 4, stride = D->xsrc_stride, total = MT * n4;
+                for (int i = blockIdx.x * kThreads + threadIdx.x; i < total; i += gridDim.x * kThreads) {
+                    const int m = i / n4, q = i - m * n4;
+                    const float4 g = ldcg4(D->xsrc + static_cast<size_t>(m) * stride + 4 * q);
+                    const float4 u = ldcg4(D->xsrc + static_cast<size_t>(m) * stride + K + 4 * q);
+                    *reinterpret_cast<uint2*>(D->aout + static_cast<size_t>(m) * K + 4 * q) =
+                        make_uint2(bf16x2_rn(silu(g.x) * u.x, silu(g.y) * u.y), bf16x2_rn(silu(g.z) * u.z, silu(g.w) * u.w));
+                }
+            }
+        }
+        if (kind_of() == kPhaseProj && !dead && t1 > t0) {
             float d[4][4] = {};
             const int NKT = P.NKT;
             const int last_len = P.K - (NKT - 1) * kKT;
@@ -1217,9 +1652,9 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                         if (P.uniform && stage) {
                             tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), kc);
                         } else if (P.uniform) {
-                            tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, kc);
+                            tile_mma_full<I8, PH>(d, tp + lane * 16, xlane + kt * kKT, kc);
                         } else {
-                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr, kc);
+                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr, kc, 0, PH && !stage);
                         }
 #endif
                         tp += rows * klen * E;

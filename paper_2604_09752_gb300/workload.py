@@ -12,7 +12,9 @@ inputs and outputs move with one host<->device copy each.
 A chained workload (``chained=True``) wires the projections into decoder layers
 (synth.workloads.chain_links): the device computes every projection's x from
 earlier outputs, so the step's only inputs are the residual stream h0 and the
-norm weights.
+norm weights.  With ``kv_len=L_max`` each layer also gets a KV cache of L_max
+positions, and O's x is attention of the new tokens over it (the step's L_past
+is a device int set by ``fill_chain``).
 """
 from __future__ import annotations
 
@@ -51,7 +53,7 @@ class DeviceWorkload:
 
     def __init__(self, wl: swl.Workload, seed: int = 0, max_M: int = 8, layout: str = "packed",
                  device: Optional[torch.device] = None, projs: Optional[List[swl.Proj]] = None,
-                 chained: bool = False):
+                 chained: bool = False, kv_len: Optional[int] = None):
         assert layout in ("packed", "rowmajor")
         self.wl = wl
         self.seed = seed
@@ -79,14 +81,22 @@ class DeviceWorkload:
         self.bufs: List[_ProjBuf] = []
         self._load_weights(offs)
         self.chained = chained
+        self.kv_len = kv_len if chained else None
         if chained:
-            self.links = swl.chain_links(swl.Workload(wl.name, wl.family, wl.wtype, wl.M, self.projs))
+            self.links = swl.chain_links(swl.Workload(wl.name, wl.family, wl.wtype, wl.M, self.projs),
+                                         attention=self.kv_len is not None)
             H = self.projs[0].K
             hb = _round(max_M * H * 4)
             # h0, the two residual buffers, then the norm weights [n_norms, H] bf16
             self.n_norms = max(l.gamma for l in self.links) + 1
             self.h_arena = torch.zeros(3 * hb + _round(self.n_norms * H * 2), dtype=torch.uint8, device=self.device)
             self._hb = hb
+        if self.kv_len is not None:
+            self.n_heads = H // swl.HEAD_DIM
+            self.attn_layers = sorted({l.layer for l in self.links if l.op == swl.XOP_ATTENTION})
+            self._kvb = _round(2 * self.n_heads * self.kv_len * swl.HEAD_DIM * 2)
+            self.kv_arena = torch.zeros(len(self.attn_layers) * self._kvb, dtype=torch.uint8, device=self.device)
+            self.lpast = torch.zeros(64, dtype=torch.int32, device=self.device)
 
     # ------------------------------------------------------------------ loading
     def _load_weights(self, offs):
@@ -145,6 +155,30 @@ class DeviceWorkload:
         torch.cuda.synchronize(self.device)
         return h0
 
+    def fill_kv(self, L_past: int):
+        """Every layer's seeded KV cache (synth.workloads.gen_kv_cache) and the step's L_past."""
+        assert self.kv_len is not None
+        n = 2 * self.n_heads * self.kv_len * swl.HEAD_DIM
+        host = torch.empty(n * 2, dtype=torch.uint8, pin_memory=True)
+        for i, layer in enumerate(self.attn_layers):
+            torch.cuda.synchronize(self.device)   # the staging buffer is reused
+            swl.gen_kv_cache(self.seed, self.wl, layer, self.kv_len, out=host.data_ptr())
+            self.kv_arena[i * self._kvb: i * self._kvb + n * 2].copy_(host, non_blocking=True)
+        self.set_lpast(L_past)
+        torch.cuda.synchronize(self.device)
+
+    def set_lpast(self, L_past: int):
+        self.lpast[0] = L_past
+
+    def kv_ptr(self, layer: int) -> int:
+        return self.kv_arena.data_ptr() + self.attn_layers.index(layer) * self._kvb
+
+    def kv(self, layer: int) -> torch.Tensor:
+        """Layer `layer`'s cache as int16 bf16 bits [2, n_heads, L_max, 128]."""
+        o = self.attn_layers.index(layer) * self._kvb
+        n = 2 * self.n_heads * self.kv_len * swl.HEAD_DIM
+        return self.kv_arena[o: o + n * 2].view(torch.int16).view(2, self.n_heads, self.kv_len, swl.HEAD_DIM)
+
     def h_ptr(self, j: int) -> int:
         """-1: the input h0; 0 / 1: the residual buffers."""
         return self.h_arena.data_ptr() + (j + 1) * self._hb
@@ -169,6 +203,9 @@ class DeviceWorkload:
             if l.op == swl.XOP_RMSNORM:
                 out.append((l.op, src, b.proj.K, 0, self.h_ptr(l.h_in), self.h_ptr(l.h_out) if l.h_out >= 0 else None,
                             self.gamma_ptr(l.gamma), swl.RMS_EPS))
+            elif l.op == swl.XOP_ATTENTION:
+                out.append((l.op, src, self.bufs[l.src].proj.N, 0, None, None, None, 0.0, self.kv_ptr(l.layer),
+                            self.lpast.data_ptr(), self.n_heads, self.kv_len))
             else:
                 out.append((l.op, src, self.bufs[l.src].proj.N, l.src_off, None, None, None, 0.0))
         return out

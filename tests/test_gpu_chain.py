@@ -2,6 +2,10 @@
 outputs of the projections before it (RMSNorm with the residual add, the V third of QKV for
 attention over one position, SwiGLU), in the same persistent launch.
 
+Attention over a KV cache (O's x in the chained step, when the workload has caches) is checked at
+the attention bar instead (relative L2 <= 1e-3, max <= 1e-2 max |x|, at most 1% of elements off by
+any ulp), and every layer's cache after the step bit for bit.
+
 Two checks, both against the fp64 oracle:
   * step by step ("teacher forced"): the oracle recomputes each projection's x from the GPU's own
     earlier outputs and the residual stream they imply, and each y from the GPU's own x.  A
@@ -55,6 +59,18 @@ def check_x(x_gpu, x_ref, op, what):
     if op == swl.XOP_SLICE:
         assert np.array_equal(x_gpu, x_ref), f"{what}: sliced x differs"
         return
+    if op == swl.XOP_ATTENTION:
+        # out = sum_j p_j v_j can cancel to values far below max |x|, where the fp32 softmax and sums
+        # (errors ~2^-24 max |v| absolute) move the bf16 rounding by several ulps: the attention bar
+        # of test_gpu_attention.py (the projections' bar) applies, with ulp flips still rare
+        g, r = bf16_values(x_gpu), bf16_values(x_ref)
+        rel = np.linalg.norm(g - r) / np.linalg.norm(r)
+        assert rel <= parity.REL_L2, f"{what}: attention x relative L2 {rel:.3e}"
+        mx = np.abs(g - r).max()
+        assert mx <= parity.MAX_REL * np.abs(r).max(), f"{what}: attention x max error {mx:.3e}"
+        flips = ordered(x_gpu) != ordered(x_ref)
+        assert flips.mean() <= 0.01, f"{what}: {flips.mean():.3%} of attention x elements differ"
+        return
     d = np.abs(ordered(x_gpu) - ordered(x_ref))
     tiny = np.abs(bf16_values(x_gpu) - bf16_values(x_ref)) <= 2.0 ** -24 * np.abs(bf16_values(x_ref)).max()
     bad = (d > 1) & ~tiny
@@ -71,14 +87,24 @@ def weights_of(dw, p, rows=None):
     return swl.gen_rows(dw.seed, dw.wl, p, rows)
 
 
-def teacher_forced(dw, M, what, rows_of=None):
-    """Check every projection of one chained step from the GPU's own earlier outputs."""
+def kv_caches(dw, L_past):
+    """The oracle's view of every layer's cache before the step: layer -> [kv bits, L_past, n_heads]."""
+    if dw.kv_len is None:
+        return None
+    return {l: [swl.gen_kv_cache(dw.seed, dw.wl, l, dw.kv_len).reshape(2, dw.n_heads, dw.kv_len, swl.HEAD_DIM),
+                L_past, dw.n_heads] for l in dw.attn_layers}
+
+
+def teacher_forced(dw, M, what, rows_of=None, L_past=None):
+    """Check every projection of one chained step from the GPU's own earlier outputs (and, with KV
+    caches, every layer's cache after the step, bit for bit)."""
     h0 = swl.gen_h0(dw.seed, dw.wl, M)
     gammas = [dw.gamma(j).cpu().numpy().view(np.uint16) for j in range(dw.n_norms)]
+    caches = kv_caches(dw, L_past)
     ys, h = [], [None, None]
     for i, (b, link) in enumerate(zip(dw.bufs, dw.links)):
         p = b.proj
-        x_ref, h_out = oracle.Oracle(oracle._l()).prep(link, ys, h, h0, gammas, swl.RMS_EPS)
+        x_ref, h_out = oracle.Oracle(oracle._l()).prep(link, ys, h, h0, gammas, swl.RMS_EPS, caches)
         if h_out is not None:
             h[link.h_out] = h_out
         x_gpu = dw.x(i, M).cpu().numpy().view(np.uint16)
@@ -96,6 +122,9 @@ def teacher_forced(dw, M, what, rows_of=None):
         last = max((i for i, l in enumerate(dw.links) if l.h_out == j), default=None)
         if last is not None:
             assert np.array_equal(dw.h(j, M).cpu().numpy().view(np.uint32), h[j].view(np.uint32)), f"{what} h{j}"
+    for layer, (kv_ref, _, _) in (caches or {}).items():
+        kv_gpu = dw.kv(layer).cpu().numpy().view(np.uint16)
+        assert np.array_equal(kv_gpu, kv_ref), f"{what}: layer {layer}'s KV cache after the step"
     return ys
 
 
@@ -107,8 +136,9 @@ def narrow_chain(wtype):
                         "two-layer narrow decoder for chained M = 4")
 
 
-@pytest.mark.parametrize("name,M", [("1b-bf16", 1), ("1b-bf16", 2), ("1b-bf16", 3), ("7b-int8", 1), ("7b-bf16", 1),
-                                    ("narrow-bf16", 4), ("narrow-int8", 4), ("narrow-bf16", 3)])
+@pytest.mark.parametrize("name,M", [("1b-bf16", 1), ("1b-bf16", 2), ("1b-bf16", 3), ("1b-bf16", 4), ("7b-int8", 1),
+                                    ("7b-bf16", 1), ("7b-bf16", 3), ("7b-int8", 2), ("narrow-bf16", 4),
+                                    ("narrow-int8", 4), ("narrow-bf16", 3)])
 def test_small_chain(aio, name, M):
     from paper_2604_09752_gb300.workload import DeviceWorkload
     if name.startswith("narrow-"):
@@ -138,6 +168,79 @@ def test_small_chain(aio, name, M):
         assert rel <= CHAIN_REL_L2, f"{name} {b.proj.name}: end-to-end relative L2 {rel:.2e}"
         assert mx <= CHAIN_MAX_REL, f"{name} {b.proj.name}: end-to-end max error {mx:.2e} of max |y|"
     print(f"{name} M={M} end-to-end drift (rel L2 / max): " + ", ".join(drift))
+    dw.close()
+
+
+@pytest.mark.parametrize("name,M,L_max,L_past", [
+    ("7b-bf16", 1, 2048, 2047),     # the paper's 2K context, 7B-class heads (32 x 128)
+    ("7b-bf16", 3, 2048, 2045),     # PLD verification of 2 drafted tokens (L = 2)
+    ("7b-int8", 2, 2048, 1000),     # ragged context, int8 weights
+    ("1b-bf16", 3, 64, 15),         # the new tokens straddle a 16-position unit; 16 heads
+    ("1b-bf16", 1, 16, 0),          # an empty cache: attention over the new token alone
+    ("narrow-int8", 4, 512, 300),   # M = 4
+])
+def test_chain_with_attention_over_kv_cache(aio, name, M, L_max, L_past):
+    """O's x is decode attention of the new tokens over each layer's KV cache, inside the persistent
+    launch (and in chain mode), checked step by step against the oracle's attention link from the
+    GPU's own QKV output; the caches afterwards hold the new tokens' k and v, bit for bit."""
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    wl = narrow_chain(name.split("-")[1]) if name.startswith("narrow-") else swl.truncated(swl.WORKLOADS[name], 2)
+    dw = DeviceWorkload(wl, seed=5, max_M=M, chained=True, kv_len=L_max)
+    dw.fill_chain(M)
+    dw.fill_kv(L_past)
+    for flags in (aio.AIO_STEP_GRAPH | aio.AIO_STEP_PERSISTENT, aio.AIO_STEP_GRAPH | aio.AIO_STEP_PDL):
+        dw.x_arena.fill_(0xFF)
+        dw.y_arena.fill_(0xFF)
+        dw.step(M, flags)
+        dw.step(M, flags)   # a second step rewrites the same cache rows with the same values
+        assert aio.aio_decode_step_check(dw.step_handle(M, flags)) == 0
+        teacher_forced(dw, M, f"{name} M={M} L={L_past + M} flags={flags}", L_past=L_past)
+    if L_past == 0 and M == 1:
+        # attention over one position returns its value vector: x of O is the V third of QKV
+        for i, l in enumerate(dw.links):
+            if l.op == swl.XOP_ATTENTION:
+                y = dw.y(l.src, M).cpu().numpy()
+                H = dw.bufs[i].proj.K
+                assert np.array_equal(dw.x(i, M).cpu().numpy().view(np.uint16), oracle.slice_x(y, 2 * H, H))
+    dw.close()
+
+
+def test_chain_attention_reports_a_short_cache(aio):
+    """L_past + M beyond the cache: the attention phases do nothing, the step completes and reports
+    device error 4; after reset, a valid L_past runs correctly again."""
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    wl = swl.truncated(swl.WORKLOADS["1b-bf16"], 1)
+    dw = DeviceWorkload(wl, seed=6, max_M=2, chained=True, kv_len=32)
+    dw.fill_chain(2)
+    dw.fill_kv(31)
+    dw.step(2)
+    with pytest.raises(aio.AioError) as e:
+        aio.aio_decode_step_check(dw.step_handle(2))
+    assert e.value.status == aio.AIO_ERR_DEVICE_TIMEOUT and "code 4" in str(e.value)
+    aio.aio_decode_step_reset(dw.step_handle(2))
+    dw.fill_kv(20)
+    dw.step(2)
+    assert aio.aio_decode_step_check(dw.step_handle(2)) == 0
+    teacher_forced(dw, 2, "after a short cache", L_past=20)
+    dw.close()
+
+
+def test_full_7b_chain_with_2k_attention_sampled(aio):
+    """The whole 7B-class chained step with attention over a 2K context in every layer (32 layers
+    and lm_head, M = 1, one persistent launch)."""
+    from paper_2604_09752_gb300.workload import DeviceWorkload
+    rng = np.random.default_rng(2)
+    dw = DeviceWorkload(swl.WORKLOADS["7b-bf16"], seed=0, max_M=1, chained=True, kv_len=2048)
+    dw.fill_chain(1)
+    dw.fill_kv(2047)
+    for _ in range(3):
+        dw.step(1)
+    assert aio.aio_decode_step_check(dw.step_handle(1)) == 0
+    assert aio.aio_decode_step_kernels(dw.step_handle(1)) == 1
+
+    def rows_of(p):
+        return np.array(sorted({0, p.N - 1, 15, 16} | set(rng.choice(p.N, 24, replace=False).tolist())))
+    teacher_forced(dw, 1, "7b chain 2K attention", rows_of, L_past=2047)
     dw.close()
 
 
@@ -182,7 +285,9 @@ def test_chained_step_rejects_bad_preparations(aio):
     proj2 = [(h2, p, p + (1 << 21), None, p + 65536)]
     proj8 = [(h8, p, p + (1 << 21), None, p + 65536)]
     cases = [
-        (proj, [(aio.AIO_X_SWIGLU, p + 4096, 2 * 11008, 0, None, None, None, 0.0)], 2, aio.AIO_ERR_UNSUPPORTED),
+        # a SwiGLU x too large to stage gets a grid-wide phase of its own; a norm that large is refused
+        (proj, [(aio.AIO_X_SWIGLU, p + 4096, 2 * 11008, 0, None, None, None, 0.0)], 2, 0),
+        (proj, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8192, None, p, 1e-5)], 2, aio.AIO_ERR_UNSUPPORTED),
         (proj2, [(9, p + 4096, 512, 0, None, None, None, 0.0)], 1, aio.AIO_ERR_INVALID_ARG),
         (proj2, [(aio.AIO_X_SLICE, None, 512, 0, None, None, None, 0.0)], 1, aio.AIO_ERR_INVALID_ARG),
         (proj2, [(aio.AIO_X_SLICE, p + 4096, 512, 300, None, None, None, 0.0)], 1, aio.AIO_ERR_INVALID_ARG),
@@ -193,8 +298,25 @@ def test_chained_step_rejects_bad_preparations(aio):
         (proj2, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8192, None, p, -1.0)], 1, aio.AIO_ERR_INVALID_ARG),
         (proj2, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8200, None, p, 1e-5)], 1, aio.AIO_ERR_ALIGNMENT),
         (proj8, [(aio.AIO_X_RMSNORM, None, 0, 0, p + 8192, None, p, 1e-5)], 5, aio.AIO_ERR_UNSUPPORTED),
+        # attention: K = 256 is 2 heads of 128
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 768, 0, None, None, None, 0.0, p + 8192, p + 64, 2, 64)], 1, 0),
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 768, 0, None, None, None, 0.0, p + 8192, p + 64, 3, 64)], 1,
+         aio.AIO_ERR_INVALID_ARG),                                                    # K != 128 n_heads
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 768, 0, None, None, None, 0.0, None, p + 64, 2, 64)], 1,
+         aio.AIO_ERR_INVALID_ARG),                                                    # no cache
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 512, 0, None, None, None, 0.0, p + 8192, p + 64, 2, 64)], 1,
+         aio.AIO_ERR_INVALID_ARG),                                                    # src_stride < 3K
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 768, 0, None, None, None, 0.0, p + 8200, p + 64, 2, 64)], 1,
+         aio.AIO_ERR_ALIGNMENT),                                                      # cache not 16-byte aligned
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 768, 0, None, None, None, 0.0, p + 8192, p + 66, 2, 64)], 1,
+         aio.AIO_ERR_ALIGNMENT),                                                      # L_past not 4-byte aligned
+        (proj2, [(aio.AIO_X_ATTENTION, p + 4096, 768, 0, None, None, None, 0.0, p + 8192, p + 64, 2, 1)], 2,
+         aio.AIO_ERR_INVALID_ARG),                                                    # L_max < M
     ]
     for pr, prep, M, status in cases:
+        if status == 0:   # a valid preparation: created (not run)
+            aio.aio_decode_step_destroy(aio.aio_decode_step_create_chained(pr, prep, M))
+            continue
         with pytest.raises(aio.AioError) as e:
             aio.aio_decode_step_create_chained(pr, prep, M)
         assert e.value.status == status, (prep, e.value)
