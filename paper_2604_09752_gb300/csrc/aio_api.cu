@@ -433,8 +433,6 @@ static aio_status validate_prep(const aio_linear* h, const aio_xprep& x, int M) 
         if (x.src_stride < 3LL * K) return fail(AIO_ERR_INVALID_ARG, "src_stride %d < 3K (%d)", x.src_stride, 3 * K);
         if (!aligned16(x.src) || !aligned16(x.kv_cache) || !aligned(x.L_past, 4) || x.src_stride % 4 != 0)
             return fail(AIO_ERR_ALIGNMENT, "src and kv_cache must be 16-byte aligned, L_past 4-byte, src_stride a multiple of 4");
-        if (aio::attn_merge_scratch(h->geo.Z) > aio::kXsBytes)
-            return fail(AIO_ERR_UNSUPPORTED, "a grid of %d warps: the attention merge lists do not fit", h->geo.Z);
         return AIO_OK;
     }
     if (x.op != AIO_X_RMSNORM && x.op != AIO_X_SWIGLU && x.op != AIO_X_SLICE)

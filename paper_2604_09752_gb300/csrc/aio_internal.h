@@ -111,9 +111,9 @@ constexpr int kAttnPos = 16;
 constexpr int kAttnUnitBytes = kAttnPos * kHeadDim * 2;
 constexpr int kAttnSlot = 2 * kAttnUnitBytes;
 constexpr int kAttnRec = 132;
-// Shared scratch of a chained step's attention merge for a grid of Z warps (it borrows the staged-x
-// area): the covering warps' record offsets and maxima, then each warp's partial sums.
-constexpr int attn_merge_scratch(int Z) { return (8 * Z + 15) / 16 * 16 + kWarps * 32 * 16 + kWarps * 4; }
+// Shared scratch of a chained step's attention merge (it borrows the staged-x area): each warp's
+// weighted sums, running max and weight.
+constexpr int kAttnMergeScratch = kWarps * 32 * 16 + kWarps * 8;
 
 // One projection of a launch; read-only while the kernel runs.  Geometry:
 //   NG  = ceil(N / 8) row groups, NKT = ceil(K / 256) tiles per group, T = NG * NKT tiles;
@@ -184,6 +184,7 @@ cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared 
 using StreamFn = void (*)(const StreamArgs);
 constexpr int kMaxChainM = 4;   // token rows of a chained step (its kernels are instantiated for M <= 4)
 static_assert(kMaxChainM < AIO_WIDE_M, "the chained step's staging limit is the narrow layout's");
+static_assert(kAttnMergeScratch <= kXsBytes, "the attention merge's scratch fits the staging area");
 StreamFn chain_stream_fn(bool i8, int M, bool phases);   // aio_chain.cu
 StreamFn chain_phase_stream_fn(bool i8, int M);          // aio_chain_ph.cu
 // chained: the chained kernels (x computed on the device); phases: with attention, merge or SwiGLU

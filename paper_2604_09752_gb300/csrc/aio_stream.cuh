@@ -370,10 +370,12 @@ struct ChunkCursor {
     IssueProj cur, nxt;
 };
 
+// Kernels with attention, merge or SwiGLU phases (PH) keep no copy of the next phase's fields:
+// they load them at the boundary instead, which frees the registers their phase code needs.
 template <bool PH>
 __device__ __forceinline__ void cursor_init(ChunkCursor& c, const StreamArgs& s, int z, int Z) {
     c.cur = load_issue<PH>(proj_desc(s, 0), s.M, Z);
-    c.nxt = s.nproj > 1 ? load_issue<PH>(proj_desc(s, 1), s.M, Z) : c.cur;
+    if constexpr (!PH) c.nxt = s.nproj > 1 ? load_issue<PH>(proj_desc(s, 1), s.M, Z) : c.cur;
     c.p = 0;
     c.t = seg(z, Z, c.cur.Tq, c.cur.Tr);
     c.te = seg(z + 1, Z, c.cur.Tq, c.cur.Tr);
@@ -387,8 +389,12 @@ __device__ __forceinline__ bool cursor_next(ChunkCursor& c, const StreamArgs& s,
     while (c.t >= c.te) {
         if (c.p + 1 >= s.nproj) return false;
         ++c.p;
-        c.cur = c.nxt;
-        if (c.p + 1 < s.nproj) c.nxt = load_issue<PH>(proj_desc(s, c.p + 1), s.M, Z);
+        if constexpr (PH) {
+            c.cur = load_issue<PH>(proj_desc(s, c.p), s.M, Z);
+        } else {
+            c.cur = c.nxt;
+            if (c.p + 1 < s.nproj) c.nxt = load_issue<PH>(proj_desc(s, c.p + 1), s.M, Z);
+        }
         c.t = seg(z, Z, c.cur.Tq, c.cur.Tr);
         c.te = seg(z + 1, Z, c.cur.Tq, c.cur.Tr);
     }
@@ -1202,10 +1208,11 @@ __device__ __forceinline__ void prep_x(const ProjDesc* d, uint16_t* xs, int xs_s
 }
 
 // The merge phase of a chained step's attention.  CTA c merges the (head, token) items c, c + G,
-// ...: the records of the warps whose units cover the head are listed in shared memory, each warp
-// adds records w, w + 8, ... weighted by 2^(max_r - max), and warp 0 adds the warps' results in
-// order (a fixed order, whatever the timing), divides by the total weight and writes the head's
-// slice of the O projection's x row as bf16.  Every warp of a CTA takes part (named barriers),
+// ...: warp w takes the records w, w + 8, ... of the warps whose units cover the head, loads them 8
+// at a time and combines them with a running maximum (each record's weighted sums rescaled by
+// 2^(max_r - max)); warp 0 then combines the 8 warps' results in order, rescaled the same way,
+// divides by the total weight and writes the head's slice of the O projection's x row as bf16.
+// The order is fixed, whatever the timing.  Every warp of a CTA takes part (named barriers),
 // whatever its state.
 template <int MT>
 __device__ __noinline__ void attn_merge(const ProjDesc* d, int Z, uint8_t* scratch, int warp, int lane) {
@@ -1214,11 +1221,9 @@ __device__ __noinline__ void attn_merge(const ProjDesc* d, int Z, uint8_t* scrat
     const int nch = (L + kAttnPos - 1) / kAttnPos;
     const int U = d->n_heads * nch, Tq = U / Z, Tr = U - Tq * Z;
     const int items = d->n_heads * MT, H = d->n_heads * kHeadDim;
-    int* srec = reinterpret_cast<int*>(scratch);
-    float* smx = reinterpret_cast<float*>(scratch + 4 * Z);
-    float4* wacc = reinterpret_cast<float4*>(scratch + (8 * Z + 15) / 16 * 16);
-    float* wl = reinterpret_cast<float*>(wacc + kWarps * 32);
-    const int tid = warp * 32 + lane;
+    float4* wacc = reinterpret_cast<float4*>(scratch);           // [kWarps][32]
+    float* wml = reinterpret_cast<float*>(wacc + kWarps * 32);    // [kWarps][2]: max, weight
+    constexpr int B = 8;   // records a warp loads at once
     for (int it = blockIdx.x; it < items; it += gridDim.x) {
         const int h = it / MT, m = it - h * MT;
         const int ua = h * nch, ub = ua + nch - 1;   // the head's units
@@ -1230,50 +1235,63 @@ __device__ __noinline__ void attn_merge(const ProjDesc* d, int Z, uint8_t* scrat
         while (zhi > 0 && seg(zhi, Z, Tq, Tr) > ub) --zhi;
         while (seg(zhi + 1, Z, Tq, Tr) <= ub) ++zhi;
         const int n = zhi - zlo + 1;
-        for (int i = tid; i < n; i += kThreads) {
-            const int zz = zlo + i, s0 = seg(zz, Z, Tq, Tr);
-            int r = -1;
-            float mxv = -INFINITY;
-            if (seg(zz + 1, Z, Tq, Tr) > s0) {   // a non-empty segment: its first or second record
-                r = ((zz * 2 + (s0 / nch == h ? 0 : 1)) * MT + m) * kAttnRec;
-                mxv = __ldcg(d->apart + r + 128);
-            }
-            srec[i] = r;
-            smx[i] = mxv;
-        }
-        named_barrier_sync();
-        float gm = -INFINITY;
-        for (int i = lane; i < n; i += 32) gm = fmaxf(gm, smx[i]);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
-        float l = 0.0f;
+        float gm = -INFINITY, gl = 0.0f;
         float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-#pragma unroll 4
-        for (int i = warp; i < n; i += kWarps) {
-            const int r = srec[i];
-            if (r < 0) continue;
-            const float w = smx[i] == -INFINITY ? 0.0f : exp2f(smx[i] - gm);
-            l = fmaf(__ldcg(d->apart + r + 129), w, l);
-            const float4 v = ldcg4(d->apart + r + 4 * lane);
-            a = make_float4(fmaf(v.x, w, a.x), fmaf(v.y, w, a.y), fmaf(v.z, w, a.z), fmaf(v.w, w, a.w));
+        for (int i0 = warp; i0 < n; i0 += B * kWarps) {
+            float rm[B], rl[B];
+            float4 rv[B];
+#pragma unroll
+            for (int b = 0; b < B; ++b) {   // the records' loads, issued together
+                const int i = i0 + b * kWarps;
+                rm[b] = -INFINITY;
+                rl[b] = 0.0f;
+                rv[b] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+                if (i < n) {
+                    const int zz = zlo + i, s0 = seg(zz, Z, Tq, Tr);
+                    if (seg(zz + 1, Z, Tq, Tr) > s0) {   // a non-empty segment: its first or second record
+                        const float* r = d->apart + ((zz * 2 + (s0 / nch == h ? 0 : 1)) * MT + m) * kAttnRec;
+                        rm[b] = __ldcg(r + 128);
+                        rl[b] = __ldcg(r + 129);
+                        rv[b] = ldcg4(r + 4 * lane);
+                    }
+                }
+            }
+#pragma unroll
+            for (int b = 0; b < B; ++b) {   // combined in record order
+                if (rm[b] == -INFINITY) continue;
+                const float nm = fmaxf(gm, rm[b]);
+                const float so = exp2f(gm - nm), sr = exp2f(rm[b] - nm);   // so = 0 while gm is -inf
+                gl = gl * so + rl[b] * sr;
+                a = make_float4(fmaf(rv[b].x, sr, a.x * so), fmaf(rv[b].y, sr, a.y * so), fmaf(rv[b].z, sr, a.z * so),
+                                fmaf(rv[b].w, sr, a.w * so));
+                gm = nm;
+            }
         }
         wacc[warp * 32 + lane] = a;
-        if (lane == 0) wl[warp] = l;
+        if (lane == 0) {
+            wml[2 * warp] = gm;
+            wml[2 * warp + 1] = gl;
+        }
         named_barrier_sync();
         if (warp == 0) {
+            float M_ = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) M_ = fmaxf(M_, wml[2 * w]);
             float lt = 0.0f;
             float4 at = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
             for (int w = 0; w < kWarps; ++w) {
-                lt += wl[w];
+                const float mw = wml[2 * w];
+                const float sw = mw == -INFINITY ? 0.0f : exp2f(mw - M_);
+                lt = fmaf(wml[2 * w + 1], sw, lt);
                 const float4 v = wacc[w * 32 + lane];
-                at = make_float4(at.x + v.x, at.y + v.y, at.z + v.z, at.w + v.w);
+                at = make_float4(fmaf(v.x, sw, at.x), fmaf(v.y, sw, at.y), fmaf(v.z, sw, at.z), fmaf(v.w, sw, at.w));
             }
             const float inv = 1.0f / lt;
             *reinterpret_cast<uint2*>(d->aout + static_cast<size_t>(m) * H + h * kHeadDim + 4 * lane) =
                 make_uint2(bf16x2_rn(at.x * inv, at.y * inv), bf16x2_rn(at.z * inv, at.w * inv));
         }
-        named_barrier_sync();   // the lists are read before the next item rewrites them
+        named_barrier_sync();   // the warps' results are read before the next item rewrites them
     }
     fence_proxy_async_smem();   // the scratch writes precede the next phase's bulk copies into this area
 }
