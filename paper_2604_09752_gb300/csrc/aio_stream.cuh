@@ -1541,6 +1541,10 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         // phase fall in different banks.
         const int xs_stride = P.K + kXsPad;
         const bool stage = kind_of() == kPhaseProj && P.M * xs_stride * 2 <= SL::kXsBytes;
+        // Plain kernels: an x that no phase of the launch writes (the host checks every buffer the
+        // step writes) was staged by this CTA's last warp at the end of the previous projection, so
+        // that its copy overlaps the grid barrier; computing still waits for the barrier.
+        const bool early = !CH && p > 0 && stage && !P.xfence;
         // Warp 0 stages x once every CTA has finished the previous projection (every warp of this
         // CTA has then finished reading the previous x and fenced its reads against async writes):
         // one bulk copy per token row.  When x may have been written by other CTAs earlier in the
@@ -1548,7 +1552,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
         // them before these async-proxy reads: in a chained step whenever x is staged as given (the
         // O projection after attention), in a plain step where the host found x aliased.
         auto stage_x = [&]() {
-            if (stage && (!CH || P.xop == kXGiven) && lane == 0) {
+            if (stage && !early && (!CH || P.xop == kXGiven) && lane == 0) {
                 if (CH || P.xfence) fence_proxy_async_all();
                 mbar_expect_tx(xbar, static_cast<uint32_t>(P.M * P.K * 2));
                 for (int m = 0; m < P.M; ++m)
@@ -1566,7 +1570,7 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                 stage_x();
                 if (lane == 0) st_release_cta_shared(&cta_sync[1], static_cast<unsigned>(p));
                 if (polled && p > 1 && blockIdx.x == 0 && lane == 0) s.done[p - 2] = 0u;   // nobody polls it any more
-            } else if (AIO_XBAR_ONLY && stage && (!CH || P.xop == kXGiven)) {
+            } else if (AIO_XBAR_ONLY && stage && !early && (!CH || P.xop == kXGiven)) {
                 // warp 0 stages x only after the grid counter is complete, so the staged x's
                 // barrier, waited on below, already orders this warp after the previous projection
                 ok = true;
@@ -1728,7 +1732,22 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             __syncwarp();
             if (lane == 0) fence_proxy_async_smem();   // this warp's reads of xs precede the next staging
         }
-        if (s.nproj > 1 && p + 1 < s.nproj) cta_arrive(&cta_sync[0], &s.done[p], lane);
+        if (s.nproj > 1 && p + 1 < s.nproj) {
+            const unsigned g = cta_arrive(&cta_sync[0], &s.done[p], lane);
+            if constexpr (!CH) {
+                if (g != 0xffffffffu && lane == 0) {
+                    // the CTA's last warp: every warp has finished (and fenced) its reads of this
+                    // projection's x, so the next one's may be staged now if nothing writes it
+                    const Proj Q = load_proj<CH>(proj_desc(s, p + 1), MT);
+                    const int qs = Q.K + kXsPad;
+                    if (Q.M * qs * 2 <= SL::kXsBytes && !Q.xfence) {
+                        mbar_expect_tx(xbar, static_cast<uint32_t>(Q.M * Q.K * 2));
+                        for (int m = 0; m < Q.M; ++m)
+                            bulk_g2s_plain(xs + m * qs, Q.x + static_cast<size_t>(m) * Q.K, static_cast<uint32_t>(Q.K * 2), xbar);
+                    }
+                }
+            }
+        }
     }
     if (s.nproj > 1) {
         const unsigned prev = cta_arrive(&cta_sync[0], s.exit_count, lane);
