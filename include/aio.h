@@ -324,7 +324,10 @@ aio_status aio_decode_step_destroy(aio_step_t step);
  *           device error word and must be zero before the first call (aio_attention_check
  *           clears it after reporting an error).  Calls sharing a workspace must not overlap.
  * Arithmetic is fp32 with an online softmax; the per-warp partial results are merged in a fixed
- * order, so results are reproducible.  Asynchronous on stream, allocates nothing.  Errors:
+ * order, so results are reproducible.  Asynchronous on stream, allocates nothing.  The two kernels
+ * launch with programmatic dependent launch: K and V start streaming before earlier work on the
+ * stream has completed, while q is read and out, the workspace and the error word are written only
+ * after it has.  Errors:
  * INVALID_ARG (NULL pointer, M outside [1, 8], L outside [M, L_max], q_stride < 128 n_heads,
  * workspace too small), UNSUPPORTED (head_dim != 128, n_heads above the grid's warp count),
  * ALIGNMENT (a pointer not 16-byte aligned, q_stride not a multiple of 4), CUDA.

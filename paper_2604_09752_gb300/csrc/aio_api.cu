@@ -873,8 +873,6 @@ extern "C" aio_status aio_attention_decode(const float* q, int q_stride, const v
     if (st != AIO_OK) return st;
     if (n_heads > sms * aio::kWarps)
         return fail(AIO_ERR_UNSUPPORTED, "n_heads=%d above %d (warps in the grid)", n_heads, sms * aio::kWarps);
-    if (sms * aio::kWarps > aio::kAttnMaxWarps)
-        return fail(AIO_ERR_UNSUPPORTED, "%d SMs: the attention merge lists at most %d warps", sms, aio::kAttnMaxWarps);
     const size_t need = aio::attn_workspace_bytes(sms * aio::kWarps, M);
     if (workspace_bytes < need) return fail(AIO_ERR_INVALID_ARG, "workspace of %zu bytes, %zu needed", workspace_bytes, need);
     AIO_CUDA(aio::launch_attention(q, q_stride, k_cache, v_cache, n_heads, L_max, L, M, out, workspace, sms,

@@ -17,6 +17,10 @@
 //     keeps a running max, sum and weighted sum of V (lane l: dims [4l, 4l + 4)).
 //   * A second small kernel merges each head's partials (max, sum, weighted V) in a fixed order, so
 //     the result does not depend on timing.
+//   * Both launch with programmatic dependent launch.  The partial kernel issues its first K and V
+//     copies (the cache does not depend on earlier work on the stream) before it waits for the
+//     previous kernel, then reads q and writes its partials; the merge kernel's small CTAs start
+//     beside it and wait for it.  So one call's merge overlaps the next call's first copies.
 #include "aio_attn.h"
 #include "aio_stream.cuh"
 
@@ -45,6 +49,7 @@ __device__ __forceinline__ long long attn_seg(long long z, long long U, int Z) {
 
 template <int MT>
 __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __grid_constant__ AttnArgs a) {
+    griddep_launch_dependents();
     extern __shared__ __align__(1024) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     uint8_t* ring = smem + warp * kAttnStages * kAttnSlot;
@@ -85,6 +90,8 @@ __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __g
         issue(i);
         ++in_flight;
     }
+    // q, the partial records and the error word wait for the previous kernel on the stream
+    griddep_wait();
 
     const float qscale = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));   // log2(e) / sqrt(d)
     float4 q4[MT];
@@ -153,18 +160,15 @@ __global__ void __launch_bounds__(kThreads, 1) aio_attn_partial_kernel(const __g
     flush();
 }
 
-// One CTA per (head, token): merges the partials of the warps whose units cover the head.  The
-// threads first list the covering warps' records and maxima in shared memory (in parallel); each
-// warp then reduces the maxima to the global max, adds the weighted sums and weighted V vectors of
-// records w, w + 8, ... (lane l: dims [4l, 4l + 4)), and warp 0 adds the 8 warps' results in order:
-// a fixed order, whatever the timing.
-constexpr int kCombineMax = kAttnMaxWarps;   // covering warps listed in shared memory
-
+// One CTA per (head, token): merges the partials of the warps whose units cover the head.  Warp w
+// takes records w, w + 8, ... (lane l: dims [4l, 4l + 4)), loads them 8 at a time and combines them
+// with a running maximum (each record's weighted sums rescaled by 2^(max_r - max)); warp 0 then
+// combines the 8 warps' results in order, rescaled the same way: one round trip for the records, in
+// a fixed order whatever the timing.
 __global__ void __launch_bounds__(kThreads) aio_attn_combine_kernel(const __grid_constant__ AttnArgs a) {
-    __shared__ long long srec[kCombineMax];
-    __shared__ float smx[kCombineMax];
+    griddep_launch_dependents();
     __shared__ float4 wacc[kWarps][32];
-    __shared__ float wl[kWarps];
+    __shared__ float wml[kWarps][2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int h = blockIdx.x / a.M, m = blockIdx.x - h * a.M;
     const long long ua = static_cast<long long>(h) * a.nch, ub = ua + a.nch - 1;   // the head's units
@@ -174,47 +178,59 @@ __global__ void __launch_bounds__(kThreads) aio_attn_combine_kernel(const __grid
     long long zhi = ub * a.Z / a.U;   // the warp holding unit ub
     while (zhi > 0 && attn_seg(zhi, a.U, a.Z) > ub) --zhi;
     while (attn_seg(zhi + 1, a.U, a.Z) <= ub) ++zhi;
-    const int n = min(static_cast<int>(zhi - zlo + 1), kCombineMax);
-    for (int i = threadIdx.x; i < n; i += kThreads) {
-        const long long zz = zlo + i;
-        const long long s0 = attn_seg(zz, a.U, a.Z);
-        long long r = -1;
-        float mx = -INFINITY;
-        if (attn_seg(zz + 1, a.U, a.Z) > s0) {   // non-empty segment
-            const int si = s0 / a.nch == h ? 0 : 1;
-            r = ((zz * 2 + si) * a.M + m) * kAttnRec;
-            mx = a.part[r + 128];
-        }
-        srec[i] = r;
-        smx[i] = mx;
-    }
-    __syncthreads();
-    float M_ = -INFINITY;
-    for (int i = lane; i < n; i += 32) M_ = fmaxf(M_, smx[i]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M_ = fmaxf(M_, __shfl_xor_sync(0xffffffffu, M_, o));
-    float l = 0.0f;
+    const int n = static_cast<int>(zhi - zlo + 1);
+    griddep_wait();   // the partial kernel has completed
+    constexpr int B = 8;   // records a warp loads at once
+    float gm = -INFINITY, gl = 0.0f;
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-#pragma unroll 4
-    for (int i = warp; i < n; i += kWarps) {
-        const long long r = srec[i];
-        if (r < 0) continue;
-        const float w = smx[i] == -INFINITY ? 0.0f : exp2f(smx[i] - M_);
-        l = fmaf(a.part[r + 129], w, l);
-        const float4 v = *reinterpret_cast<const float4*>(a.part + r + 4 * lane);
-        acc = make_float4(fmaf(v.x, w, acc.x), fmaf(v.y, w, acc.y), fmaf(v.z, w, acc.z), fmaf(v.w, w, acc.w));
+    for (int i0 = warp; i0 < n; i0 += B * kWarps) {
+        float rm[B], rl[B];
+        float4 rv[B];
+#pragma unroll
+        for (int b = 0; b < B; ++b) {   // the records' loads, issued together
+            const int i = i0 + b * kWarps;
+            rm[b] = -INFINITY;
+            rl[b] = 0.0f;
+            rv[b] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (i < n) {
+                const long long zz = zlo + i, s0 = attn_seg(zz, a.U, a.Z);
+                if (attn_seg(zz + 1, a.U, a.Z) > s0) {   // a non-empty segment: its first or second record
+                    const float* r = a.part + ((zz * 2 + (s0 / a.nch == h ? 0 : 1)) * a.M + m) * kAttnRec;
+                    rm[b] = r[128];
+                    rl[b] = r[129];
+                    rv[b] = *reinterpret_cast<const float4*>(r + 4 * lane);
+                }
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < B; ++b) {   // combined in record order
+            if (rm[b] == -INFINITY) continue;
+            const float nm = fmaxf(gm, rm[b]);
+            const float so = exp2f(gm - nm), sr = exp2f(rm[b] - nm);   // so = 0 while gm is -inf
+            gl = gl * so + rl[b] * sr;
+            acc = make_float4(fmaf(rv[b].x, sr, acc.x * so), fmaf(rv[b].y, sr, acc.y * so), fmaf(rv[b].z, sr, acc.z * so),
+                              fmaf(rv[b].w, sr, acc.w * so));
+            gm = nm;
+        }
     }
     wacc[warp][lane] = acc;
-    if (lane == 0) wl[warp] = l;
+    if (lane == 0) {
+        wml[warp][0] = gm;
+        wml[warp][1] = gl;
+    }
     __syncthreads();
     if (warp == 0) {
+        float M_ = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) M_ = fmaxf(M_, wml[w][0]);
         float lt = 0.0f;
         float4 at = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
         for (int w = 0; w < kWarps; ++w) {
-            lt += wl[w];
+            const float sw = wml[w][0] == -INFINITY ? 0.0f : exp2f(wml[w][0] - M_);
+            lt = fmaf(wml[w][1], sw, lt);
             const float4 v = wacc[w][lane];
-            at = make_float4(at.x + v.x, at.y + v.y, at.z + v.z, at.w + v.w);
+            at = make_float4(fmaf(v.x, sw, at.x), fmaf(v.y, sw, at.y), fmaf(v.z, sw, at.z), fmaf(v.w, sw, at.w));
         }
         const float inv = 1.0f / lt;
         *reinterpret_cast<float4*>(a.out + static_cast<size_t>(m) * a.n_heads * kHeadDim + h * kHeadDim + 4 * lane) =
@@ -275,11 +291,22 @@ cudaError_t launch_attention(const float* q, int q_stride, const void* k, const 
     a.nch = (L + kAttnPos - 1) / kAttnPos;
     a.U = static_cast<long long>(n_heads) * a.nch;
     a.wait_limit_ns = wait_limit_ns;
-    f<<<grid, kThreads, kAttnSmem, s>>>(a);
-    e = cudaGetLastError();
+    // both with programmatic dependent launch (see the top of this file)
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kAttnSmem;
+    cfg.stream = s;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, f, a);
     if (e != cudaSuccess) return e;
-    aio_attn_combine_kernel<<<n_heads * M, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    cfg.gridDim = dim3(static_cast<unsigned>(n_heads * M));
+    cfg.dynamicSmemBytes = 0;
+    return cudaLaunchKernelEx(&cfg, aio_attn_combine_kernel, a);
 }
 
 }  // namespace aio

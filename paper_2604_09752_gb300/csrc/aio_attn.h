@@ -6,8 +6,6 @@
 
 namespace aio {
 
-constexpr int kAttnMaxWarps = 1536;   // warps in the grid the merge kernel can list (host-checked)
-
 // Workspace bytes for Z warps and M tokens: a 256-byte header (the device error word), then the
 // per-warp partial results.
 size_t attn_workspace_bytes(int Z, int M);

@@ -46,4 +46,7 @@ def test_partition_facts(n_heads, L):
         # them are skipped by the merge)
         nonempty = [z for z in range(zlo, zhi + 1) if seg(z + 1, U) > seg(z, U)]
         assert nonempty == heads_of[h]
-        assert zhi - zlo + 1 <= 1536                # the merge lists at most this many warps
+        for z in nonempty:                          # the record the merge reads is the one the warp wrote
+            first = seg(z, U) // nch
+            rec = 0 if first == h else 1
+            assert rec == sorted({u // nch for u in range(seg(z, U), seg(z + 1, U))}).index(h)
