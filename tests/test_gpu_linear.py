@@ -62,7 +62,7 @@ class Linear:
         self.aio.aio_linear_destroy(self.h)
 
 
-SHAPES = [(16, 1), (48, 13), (272, 9), (1040, 37), (2048, 2048), (4096, 100), (5632, 24), (11008, 40)]
+SHAPES = [(16, 1), (48, 13), (272, 9), (1040, 37), (2048, 2048), (4096, 100), (5632, 24), (11008, 40), (11008, 64)]
 
 
 @pytest.mark.parametrize("wt", ["bf16", "int8"])
