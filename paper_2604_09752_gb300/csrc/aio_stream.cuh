@@ -43,6 +43,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "aio_internal.h"
 
 namespace aio {
@@ -1648,69 +1650,80 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
             const int xtok = min(tok, MT - 1);   // full tiles: lanes of tokens >= M read token M-1's x
             [[maybe_unused]] const uint16_t* xlane = P.x + static_cast<size_t>(xtok) * P.K + 8 * (lane & 3);
             const uint32_t xs_lane = smem_addr(xs) + static_cast<uint32_t>((xtok * xs_stride + 8 * (lane & 3)) * 2);
-            while (t < tend) {
-                if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
-                    if (lane == 0) atomicExch(s.err, kDevErrTimeout);
-                    dead = true;
-                    break;
-                }
-                const int nt = min(C, tend - t);
-                const uint8_t* tp = ring + cslot * TL::kSlot;
+            // The tile loop, compiled twice: FAST is the common case (every tile full, x staged), with
+            // the tile shape, the x source and the row count known at compile time, so each tile
+            // carries fewer branches; the general copy takes ragged, row-major and unstaged tiles.
+            auto consume = [&](auto fast_tag) {
+                constexpr bool FAST = decltype(fast_tag)::value;
+                while (t < tend) {
+                    if (!__all_sync(0xffffffffu, mbar_wait(&bars[cslot], cphase, s.wait_limit_ns))) {
+                        if (lane == 0) atomicExch(s.err, kDevErrTimeout);
+                        dead = true;
+                        break;
+                    }
+                    const int nt = min(C, tend - t);
+                    const uint8_t* tp = ring + cslot * TL::kSlot;
 #pragma unroll
-                for (int j = 0; j < C; ++j) {
-                    if (j < nt) {
-                        const int klen = kt == NKT - 1 ? last_len : kKT;
+                    for (int j = 0; j < C; ++j) {
+                        if (j < nt) {
+                            const int klen = FAST ? kKT : (kt == NKT - 1 ? last_len : kKT);
 #if AIO_FFMA
-                        if (P.uniform && stage) {
-                            ffma_full_s<I8, MT>(d, smem_addr(tp) + lane * 16,
-                                                smem_addr(xs) + 16 * (lane & 3) + kt * (kKT * 2), xs_stride * 2);
-                        } else if (P.uniform) {
-                            ffma_full_g<I8, MT>(d, tp + lane * 16, P.x + 8 * (lane & 3) + kt * kKT, P.K);
-                        } else {
-                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, stage ? xs : P.x, kc,
-                                         stage ? xs_stride : P.K);
-                        }
-#else
-                        if (P.uniform && stage) {
-                            tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), kc);
-                        } else if (P.uniform) {
-                            tile_mma_full<I8, PH>(d, tp + lane * 16, xlane + kt * kKT, kc);
-                        } else {
-                            tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr, kc, 0, PH && !stage);
-                        }
-#endif
-                        tp += rows * klen * E;
-                        if (kt == NKT - 1 || t == tend - 1) {
-                            float sum[4];
-#if AIO_FFMA
-                            ffma_finish<MT>(d, sum, lane);
-#else
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
-#endif
-                            if (!finish_group<I8, MT>(P, s, Z, sum, g, rows, z, t0, t1, lane)) {
-                                if (lane == 0) atomicCAS(s.err, 0, kDevErrTimeout);
-                                dead = true;
+                            if (FAST || (P.uniform && stage)) {
+                                ffma_full_s<I8, MT>(d, smem_addr(tp) + lane * 16,
+                                                    smem_addr(xs) + 16 * (lane & 3) + kt * (kKT * 2), xs_stride * 2);
+                            } else if (P.uniform) {
+                                ffma_full_g<I8, MT>(d, tp + lane * 16, P.x + 8 * (lane & 3) + kt * kKT, P.K);
+                            } else {
+                                tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, stage ? xs : P.x, kc,
+                                             stage ? xs_stride : P.K);
                             }
+#else
+                            if (FAST || (P.uniform && stage)) {
+                                tile_mma_full_s<I8>(d, smem_addr(tp) + lane * 16, xs_lane + kt * (kKT * 2), kc);
+                            } else if (P.uniform) {
+                                tile_mma_full<I8, PH>(d, tp + lane * 16, xlane + kt * kKT, kc);
+                            } else {
+                                tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow_ptr, kc, 0, PH && !stage);
+                            }
+#endif
+                            tp += FAST ? TL::kBytes : rows * klen * E;
+                            if (kt == NKT - 1 || t == tend - 1) {
+                                float sum[4];
+#if AIO_FFMA
+                                ffma_finish<MT>(d, sum, lane);
+#else
 #pragma unroll
-                            for (int q = 0; q < 4; ++q)
+                                for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
+#endif
+                                if (!finish_group<I8, MT>(P, s, Z, sum, g, FAST ? kRows : rows, z, t0, t1, lane)) {
+                                    if (lane == 0) atomicCAS(s.err, 0, kDevErrTimeout);
+                                    dead = true;
+                                }
 #pragma unroll
-                                for (int i = 0; i < 4; ++i) d[q][i] = 0.0f;
-                        }
-                        ++t;
-                        if (++kt == NKT) {
-                            kt = 0;
-                            ++g;
-                            rows = min(kRows, P.N - g * kRows);
+                                for (int q = 0; q < 4; ++q)
+#pragma unroll
+                                    for (int i = 0; i < 4; ++i) d[q][i] = 0.0f;
+                            }
+                            ++t;
+                            if (++kt == NKT) {
+                                kt = 0;
+                                ++g;
+                                if (!FAST) rows = min(kRows, P.N - g * kRows);
+                            }
                         }
                     }
+                    // Every lane's reads of the slot have returned (their values fed the MMAs above), so
+                    // lane 0 may let the bulk copy overwrite it, as a consumer release would.
+                    __syncwarp();
+                    cslot = (cslot + 1 == S) ? 0 : cslot + 1;
+                    cphase ^= (cslot == 0) ? 1u : 0u;
+                    refill(p);
                 }
-                // Every lane's reads of the slot have returned (their values fed the MMAs above), so
-                // lane 0 may let the bulk copy overwrite it, as a consumer release would.
-                __syncwarp();
-                cslot = (cslot + 1 == S) ? 0 : cslot + 1;
-                cphase ^= (cslot == 0) ? 1u : 0u;
-                refill(p);
+            };
+            if (P.uniform && stage) {
+                consume(std::true_type{});
+            } else {
+                consume(std::false_type{});
             }
             if (!dead) {
                 while (ahead < TL::kAhead && in_flight < S && issue_next()) {
