@@ -12,7 +12,8 @@
 //   * Rings.  One CTA per SM; each warp owns a shared-memory ring of slots.  Lane 0 issues one
 //     cp.async.bulk per slot (global -> shared, L2 evict-first) completing on the slot's mbarrier;
 //     the warp waits (bounded by %globaltimer), computes, and refills the slot.  The issue cursor
-//     runs ahead across projection boundaries: weights never depend on x.
+//     runs ahead across projection boundaries: weights never depend on x.  Plain launches of
+//     M >= AIO_WIDE_M (two slots per warp) read a slot into registers and refill it before computing.
 //   * x.  Once per CTA and projection, warp 0 stages x into shared memory (one bulk copy per token
 //     row, rows padded by 64 B) when it fits; otherwise the lanes read x from global memory.
 //   * Arithmetic on the tensor cores: mma.sync.m16n8k16, bf16 in, fp32 accumulate, with A = W
@@ -1663,6 +1664,54 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                     }
                     const int nt = min(C, tend - t);
                     const uint8_t* tp = ring + cslot * TL::kSlot;
+#if !AIO_FFMA
+                    if constexpr (FAST && !CH && MT >= AIO_WIDE_M) {
+                        // Early release (plain launches of M >= AIO_WIDE_M, whose rings have two slots):
+                        // read the slot's tiles of W into registers and hand the slot back to the
+                        // issuing lane before the arithmetic, so that its next copy is in flight while
+                        // these tiles are computed.  Every lane's reads are ordered before lane 0's
+                        // copy by the warp barrier and the proxy fence.
+                        uint4 wr[C][TL::kPieces];
+                        const uint32_t wa = smem_addr(tp) + lane * 16;
+#pragma unroll
+                        for (int j = 0; j < C; ++j)
+#pragma unroll
+                            for (int q = 0; q < TL::kPieces; ++q) wr[j][q] = lds128(wa + j * TL::kBytes + q * 512);
+                        __syncwarp();
+                        if (lane == 0) fence_proxy_async_smem();
+                        cslot = (cslot + 1 == S) ? 0 : cslot + 1;
+                        cphase ^= (cslot == 0) ? 1u : 0u;
+                        refill(p);
+#pragma unroll
+                        for (int j = 0; j < C; ++j) {
+                            if (j < nt) {
+                                uint4 xv[kRuns];
+#pragma unroll
+                                for (int u = 0; u < kRuns; ++u) xv[u] = lds128(xs_lane + kt * (kKT * 2) + 64 * u);
+                                tile_mma_frag<I8>(d, wr[j], xv, kc);
+                                if (kt == NKT - 1 || t == tend - 1) {
+                                    float sum[4];
+#pragma unroll
+                                    for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
+                                    if (!finish_group<I8, MT>(P, s, Z, sum, g, kRows, z, t0, t1, lane)) {
+                                        if (lane == 0) atomicCAS(s.err, 0, kDevErrTimeout);
+                                        dead = true;
+                                    }
+#pragma unroll
+                                    for (int q = 0; q < 4; ++q)
+#pragma unroll
+                                        for (int i = 0; i < 4; ++i) d[q][i] = 0.0f;
+                                }
+                                ++t;
+                                if (++kt == NKT) {
+                                    kt = 0;
+                                    ++g;
+                                }
+                            }
+                        }
+                        continue;
+                    }
+#endif
 #pragma unroll
                     for (int j = 0; j < C; ++j) {
                         if (j < nt) {
