@@ -309,9 +309,9 @@ def step_record(name, M, wtype, wbytes, ms, peak, launches, **extra):
 def bench_single_linear(args, peak):
     """The single 2048 x 2048 bf16 layer at M = 1 (8.39 MB: it would sit in the 129 MB L2 if timed
     alone), timed over 64 distinct seeded copies (537 MB, over 4x L2) so that every launch streams
-    from HBM.  Each copy is one standalone launch of the single-projection kernel (what
-    aio_linear_run enqueues), the 64 chained with programmatic dependent launch in one CUDA graph;
-    the time per layer is the graph's time / 64."""
+    from HBM.  Each copy is one standalone launch of the small-projection kernel (what
+    aio_linear_run enqueues for this shape: one CTA per row group), the 64 chained with programmatic
+    dependent launch in one CUDA graph; the time per layer is the graph's time / 64."""
     from paper_2604_09752_gb300 import aio
     from paper_2604_09752_gb300.workload import DeviceWorkload
     from synth import workloads as swl
@@ -333,6 +333,7 @@ def bench_single_linear(args, peak):
     return {"workload": "linear-2048", "baseline_config": 1, "M": 1, "wtype": "bf16", "weight_bytes_per_layer": layer,
             "ms_per_layer": round(per, 5), "GB/s": round(gbs, 2), "frac_of_measured_peak": round(gbs / peak, 4),
             "copies": copies, "rotating_weight_bytes": copies * layer, "launches_per_layer": 1,
+            "kernel": "aio_small_kernel<1, bf16> (one CTA per row group)",
             "l2": "64 distinct copies, 537 MB, over 4x the 129 MB L2"}
 
 

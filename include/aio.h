@@ -69,6 +69,7 @@ typedef enum {
 /* aio_linear_create flags */
 #define AIO_FLAG_ROWMAJOR   0x1u   /* aio_linear_run reads W as plain row-major [N, K] (no packing) */
 #define AIO_FLAG_NO_PDL     0x2u   /* launch without programmatic dependent launch */
+#define AIO_FLAG_STREAM_KERNEL 0x4u /* aio_linear_run always takes the stream kernel (never the small-projection launch) */
 #define AIO_FLAG_TEST_STALL 0x100u /* TEST ONLY: the grid's last warp skips its first weight copy,
                                       so its bounded wait (20 ms) expires and the run reports
                                       AIO_ERR_DEVICE_TIMEOUT; outputs are then undefined */
@@ -207,13 +208,23 @@ aio_status aio_linear_unpack(aio_linear_t h, const void* W_packed, void* W_rowma
  * Uses the handle's workspace: runs of one handle must not overlap in time (issue them on
  * one stream, or order the streams).  With PDL (default) the kernel may start streaming W
  * while the previous kernel on the stream is still running; it reads x and writes y only
- * after that kernel has completed.  Errors: INVALID_ARG, ALIGNMENT, STATE, CUDA.
+ * after that kernel has completed.
+ * Two launches (Sec. 3.1: a projection launched on its own is bound by latency once its weights
+ * are a few MB).  A small packed projection -- at most 2 x (SM count) row groups of 16 rows, and
+ * K <= 2048 (bf16) or K <= 6144 (int8) -- runs as one CTA of 8 warps per row group: the warps split
+ * the group's tiles, their partial sums meet in shared memory and are added in warp order, and two
+ * such CTAs fit an SM, so a PDL launch loads its weights beside the previous one.  Every other
+ * projection, and every handle created with AIO_FLAG_STREAM_KERNEL, takes the stream kernel (all
+ * SMs, equal bytes per warp).  A decode step's per-projection launches (without
+ * AIO_STEP_PERSISTENT, and without computed x) make the same choice.
+ * Errors: INVALID_ARG, ALIGNMENT, STATE, CUDA.
  */
 aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, const void* W,
                           const void* scales, float* y, void* stream);
 
 /*
- * y = x W^T as aio_linear_run computes it, without a handle and without allocating anything.
+ * y = x W^T as the stream kernel computes it (aio_linear_run with AIO_FLAG_STREAM_KERNEL), without
+ * a handle and without allocating anything.
  * The paper has no counterpart: this is a library entry for callers that cannot allocate device
  * memory where they call -- a serving engine that has handed nearly all of HBM to its own pools
  * (weights, KV cache), so that a cudaMalloc there fails, or a hot loop in which cudaMalloc /

@@ -35,6 +35,7 @@ AIO_W_BF16 = 0
 AIO_W_INT8_PERCHANNEL = 1
 AIO_FLAG_ROWMAJOR = 0x1
 AIO_FLAG_NO_PDL = 0x2
+AIO_FLAG_STREAM_KERNEL = 0x4
 AIO_FLAG_TEST_STALL = 0x100
 AIO_STEP_GRAPH = 0x1
 AIO_STEP_PDL = 0x2

@@ -17,7 +17,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libaio.so")
 STAMP = os.path.join(HERE, "_build", "defines.txt")
-SOURCES = ["aio_gemv.cu", "aio_chain.cu", "aio_chain_ph.cu", "aio_attn.cu", "aio_pld.cu", "aio_pack.cu", "aio_api.cu"]
+SOURCES = ["aio_gemv.cu", "aio_chain.cu", "aio_chain_ph.cu", "aio_attn.cu", "aio_small.cu", "aio_pld.cu", "aio_pack.cu",
+           "aio_api.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

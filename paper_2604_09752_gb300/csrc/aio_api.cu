@@ -22,7 +22,7 @@ namespace {
 
 constexpr uint32_t kLinearMagic = 0xA10113EAu;
 constexpr uint32_t kStepMagic = 0xA1057E90u;
-constexpr unsigned kCreateFlags = AIO_FLAG_ROWMAJOR | AIO_FLAG_NO_PDL | AIO_FLAG_TEST_STALL;
+constexpr unsigned kCreateFlags = AIO_FLAG_ROWMAJOR | AIO_FLAG_NO_PDL | AIO_FLAG_STREAM_KERNEL | AIO_FLAG_TEST_STALL;
 constexpr unsigned kStepFlags = AIO_STEP_GRAPH | AIO_STEP_PDL | AIO_STEP_PERSISTENT;
 constexpr unsigned long long kWaitLimitNs = 1000000000ull;      // 1 s: a healthy wait takes microseconds
 constexpr unsigned long long kTestWaitLimitNs = 20000000ull;    // 20 ms for AIO_FLAG_TEST_STALL
@@ -108,6 +108,7 @@ struct aio_linear {
     unsigned flags;
     int device;
     aio::Geometry geo;
+    aio::SmallGeometry small;   // small.ok: aio_linear_run launches one CTA per row group (aio_small.cu)
     void* ws;            // partial-sum slots, then the error word
     size_t ws_bytes;
     float* partial;      // partial-sum slots (empty pattern 0xFF at rest)
@@ -125,6 +126,7 @@ struct aio_step {
     int grid;
     std::vector<aio::StreamArgs> chain;  // per-projection launches (chain mode)
     std::vector<char> chain_i8;
+    std::vector<aio::SmallGeometry> chain_small;   // chain mode: per-launch small-projection geometry
     aio::StreamArgs whole;               // one launch over the device descriptor array (persistent mode)
     void* ws;                            // workspaces, descriptors, done counters, error words
     size_t ws_bytes;
@@ -275,6 +277,8 @@ aio_status aio_linear_create(aio_linear_t* out, int K, int N, aio_wtype wt, int 
     h->flags = flags;
     h->device = dev;
     h->geo = geo;
+    h->small = aio::small_geometry(K, N, wt == AIO_W_INT8_PERCHANNEL, (flags & AIO_FLAG_ROWMAJOR) != 0, sms);
+    if (flags & AIO_FLAG_STREAM_KERNEL) h->small.ok = false;
     h->ws = mem;
     h->ws_bytes = ws + 256;
     h->partial = static_cast<float*>(mem);
@@ -295,9 +299,9 @@ aio_status aio_linear_packed_bytes(aio_linear_t h, size_t* w_bytes, size_t* scal
 aio_status aio_linear_launch_info(aio_linear_t h, int* grid, int* block, size_t* smem_bytes, long long* tiles) {
     aio_status st = valid_linear(h);
     if (st != AIO_OK) return st;
-    if (grid) *grid = h->geo.grid;
+    if (grid) *grid = h->small.ok ? h->small.grid : h->geo.grid;
     if (block) *block = aio::kThreads;
-    if (smem_bytes) *smem_bytes = aio::kSmemBytes;
+    if (smem_bytes) *smem_bytes = h->small.ok ? h->small.smem : static_cast<size_t>(aio::kSmemBytes);
     if (tiles) *tiles = h->geo.T;
     return AIO_OK;
 }
@@ -345,8 +349,12 @@ aio_status aio_linear_run(aio_linear_t h, const void* x, int M, int K, int N, co
     if ((st = validate_run(h, x, M, W, scales, y)) != AIO_OK) return st;
     if ((st = check_device(h->device)) != AIO_OK) return st;
     const aio::StreamArgs a = single_args(h, make_desc(h, x, W, scales, y, h->partial), M, h->err);
-    AIO_CUDA(aio::launch_stream(a, h->wt == AIO_W_INT8_PERCHANNEL, h->geo.grid, static_cast<cudaStream_t>(stream),
-                                !(h->flags & AIO_FLAG_NO_PDL), false));
+    const bool i8 = h->wt == AIO_W_INT8_PERCHANNEL, pdl = !(h->flags & AIO_FLAG_NO_PDL);
+    if (h->small.ok) {
+        AIO_CUDA(aio::launch_small(a, i8, h->small, static_cast<cudaStream_t>(stream), pdl));
+    } else {
+        AIO_CUDA(aio::launch_stream(a, i8, h->geo.grid, static_cast<cudaStream_t>(stream), pdl, false));
+    }
     return AIO_OK;
 }
 
@@ -411,7 +419,11 @@ static aio_status step_launch_all(aio_step* s, cudaStream_t stream) {
     }
     for (int i = 0; i < s->n; ++i) {
         const bool pdl = i > 0 && (s->flags & AIO_STEP_PDL);
-        AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false, s->chained, s->phases));
+        if (s->chain_small[i].ok) {
+            AIO_CUDA(aio::launch_small(s->chain[i], s->chain_i8[i] != 0, s->chain_small[i], stream, pdl));
+        } else {
+            AIO_CUDA(aio::launch_stream(s->chain[i], s->chain_i8[i] != 0, s->grid, stream, pdl, false, s->chained, s->phases));
+        }
     }
     return AIO_OK;
 }
@@ -585,6 +597,7 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
                 s->chain.push_back(aio::StreamArgs{});
                 s->chain.back() = single_args(p.h, a, M, s->errs + e);
                 s->chain_i8.push_back(i8 ? 1 : 0);
+                s->chain_small.push_back(aio::SmallGeometry{});
             }
         }
         const bool own = preps && swiglu_phase(p.h, preps[i], M);
@@ -600,11 +613,14 @@ static aio_status step_create(aio_step_t* out, const aio_proj* projs, const aio_
             descs.push_back(g);
             s->chain.push_back(single_args(p.h, g, M, s->errs + (descs.size() - 1)));
             s->chain_i8.push_back(i8 ? 1 : 0);
+            s->chain_small.push_back(aio::SmallGeometry{});
         }
         descs.push_back(make_desc(p.h, p.x, p.W, p.scales, p.y, reinterpret_cast<float*>(base + offs[i])));
         if (preps) apply_prep(descs.back(), preps[i], own);
         s->chain.push_back(single_args(p.h, descs.back(), M, s->errs + (descs.size() - 1)));
         s->chain_i8.push_back(i8 ? 1 : 0);
+        // a plain projection of a step without computed x: the small-projection launch if it qualifies
+        s->chain_small.push_back(chained ? aio::SmallGeometry{} : p.h->small);
     }
     // A projection whose x overlaps a buffer an earlier phase of the step writes (y, a computed x, a
     // residual stream, an attention or SwiGLU output, a KV cache) reads data written in the same
@@ -772,7 +788,8 @@ aio_status aio_probe_read(const void* buf, size_t bytes, unsigned* out, void* st
 }  // extern "C"
 
 // ---------------------------------------------------------------------------------------------
-// aio_linear_run_noalloc: the single-projection launch of aio_linear_run with its cross-warp
+// aio_linear_run_noalloc: the stream kernel's single-projection launch (aio_linear_run's launch for
+// a handle created with AIO_FLAG_STREAM_KERNEL) with its cross-warp
 // scratch (partial sums of row groups split between warps) in one static
 // device array that is part of the library image, instead of a handle's cudaMalloc'd workspace.
 // It is for callers that cannot allocate device memory where they call: a serving engine that has

@@ -98,7 +98,8 @@ cudaError_t prepare_kernels() {
             }
         }
     }
-    return cudaFuncSetAttribute(aio_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    const cudaError_t e = cudaFuncSetAttribute(aio_probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    return e != cudaSuccess ? e : prepare_small_kernels();
 }
 
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop, bool chained,

@@ -192,6 +192,17 @@ StreamFn chain_phase_stream_fn(bool i8, int M);          // aio_chain_ph.cu
 cudaError_t launch_stream(const StreamArgs& a, bool i8, int grid, cudaStream_t s, bool pdl, bool coop,
                           bool chained = false, bool phases = false);
 cudaError_t occupancy(bool i8, int M, bool chained, bool phases, int* blocks_per_sm);
+// A projection small enough to launch as one CTA per row group (aio_small.cu): packed weights, at most
+// two CTAs per SM, at most 96 KB of weights per CTA (bf16 K <= 2048, int8 K <= 6144).
+struct SmallGeometry {
+    bool ok;       // the shape qualifies
+    int grid;      // CTAs: one per row group
+    int tpw;       // tiles per warp: ceil(NKT / 8)
+    size_t smem;   // dynamic shared memory per CTA
+};
+SmallGeometry small_geometry(int K, int N, bool i8, bool rowmajor, int num_sms);
+cudaError_t prepare_small_kernels();
+cudaError_t launch_small(const StreamArgs& a, bool i8, const SmallGeometry& g, cudaStream_t s, bool pdl);
 cudaError_t launch_pack(const void* src, void* dst, int N, int K, int esize, bool inverse, cudaStream_t s);
 cudaError_t launch_probe(const void* buf, long long pages, unsigned* out, int grid, cudaStream_t s);
 

@@ -1,7 +1,9 @@
 """GPU parity of one linear layer through the C ABI: y = x W^T (Sec. 2.1), int8 with per-channel
 scales (Sec. 2.4), every width M = 1..8 the API accepts (Sec. 4.2 verification rows), packed and
 row-major weights, ragged shapes, and the int8 code -128 (outside the symmetric range the recipe
-draws, but a valid code the kernel must convert exactly)."""
+draws, but a valid code the kernel must convert exactly).  Both launches of aio_linear_run are
+covered: the small-projection launch (one CTA per row group) that small packed shapes take by
+default, and the stream kernel (every other shape, and any handle with AIO_FLAG_STREAM_KERNEL)."""
 import numpy as np
 import pytest
 import torch
@@ -62,16 +64,33 @@ class Linear:
         self.aio.aio_linear_destroy(self.h)
 
 
+def n_sms():
+    return torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def small_grid(K, N, wt):
+    """The grid of the small-projection launch (one CTA per row group), or None if the shape does
+    not qualify: at most 2 x SMs row groups and at most 96 KB of weights per CTA (8 warps, each
+    ceil(NKT / 8) tiles of 8 KB bf16 or 4 KB int8)."""
+    NG, NKT = -(-N // 16), -(-K // 256)
+    tile = 4096 if wt == "int8" else 8192
+    return NG if NG <= 2 * n_sms() and 8 * -(-NKT // 8) * tile <= 96 * 1024 else None
+
+
 SHAPES = [(16, 1), (48, 13), (272, 9), (1040, 37), (2048, 2048), (4096, 100), (5632, 24), (11008, 40), (11008, 64)]
 
 
 @pytest.mark.parametrize("wt", ["bf16", "int8"])
 @pytest.mark.parametrize("K,N", SHAPES)
 @pytest.mark.parametrize("M", [1, 2, 3, 4, 5, 6, 7, 8])
-@pytest.mark.parametrize("layout_", ["packed", "rowmajor"])
+@pytest.mark.parametrize("layout_", ["packed", "packed-stream", "rowmajor"])
 def test_linear_parity(aio, wt, K, N, M, layout_):
     x, W, s = make_inputs(K, N, M, wt)
-    lin = Linear(aio, W, s, max_M=8, rowmajor=(layout_ == "rowmajor"))
+    lin = Linear(aio, W, s, max_M=8, rowmajor=(layout_ == "rowmajor"),
+                 flags=aio.AIO_FLAG_STREAM_KERNEL if layout_ == "packed-stream" else 0)
+    grid = aio.aio_linear_launch_info(lin.h)["grid"]
+    want = small_grid(K, N, wt) if layout_ == "packed" else None   # None: the stream kernel, one CTA per SM
+    assert grid == (want if want is not None else n_sms()), (grid, want)
     xd = dev(x)
     guard = 64
     yd = torch.full((M * N + 2 * guard,), 12345.0, dtype=torch.float32, device="cuda")
@@ -234,11 +253,15 @@ def test_argument_errors_launch_nothing(aio):
     lin2.close()
 
 
-def test_bounded_wait_reports_timeout_and_context_survives(aio):
+@pytest.mark.parametrize("kernel", ["small", "stream"])
+def test_bounded_wait_reports_timeout_and_context_survives(aio, kernel):
     # AIO_FLAG_TEST_STALL: one warp never receives its first tile; its wait gives up after 20 ms,
     # the kernel returns, and the host reads AIO_ERR_DEVICE_TIMEOUT.  The context stays usable.
     x, W, _ = make_inputs(2048, 512, 1, "bf16", tag=11)
-    stall = Linear(aio, W, None, max_M=1, flags=aio.AIO_FLAG_TEST_STALL)
+    extra = aio.AIO_FLAG_STREAM_KERNEL if kernel == "stream" else 0
+    assert small_grid(2048, 512, "bf16") == 32
+    stall = Linear(aio, W, None, max_M=1, flags=aio.AIO_FLAG_TEST_STALL | extra)
+    assert aio.aio_linear_launch_info(stall.h)["grid"] == (32 if kernel == "small" else n_sms())
     y = torch.empty(512, dtype=torch.float32, device="cuda")
     stall.run(dev(x), 1, y)
     with pytest.raises(aio.AioError) as e:

@@ -4,7 +4,8 @@ the device).  Its scratch is a static device array inside the library, and nothi
 
 Each case runs two calls in a row on one stream (the second reuses the scratch the first left) and
 checks both against the fp64 oracle at the linear-layer bar (parity.check), and bit for bit against
-aio_linear_run on the same inputs: the launch, the partition and the summation order are the same.
+aio_linear_run of a handle created with AIO_FLAG_STREAM_KERNEL on the same inputs: the launch, the
+partition and the summation order are the same.
 
 The file name sorts last so the test also runs after every other GPU test in one session."""
 import numpy as np
@@ -37,8 +38,9 @@ def _inputs(K, N, M, wt):
 
 
 def _weights(aio, W, s, K, N, M, wt_c, flags):
-    """A handle (for the aio_linear_run comparison and the packer) and the device weights."""
-    h = aio.aio_linear_create(K, N, wt_c, M, flags)
+    """A handle (for the aio_linear_run comparison and the packer) and the device weights.  The
+    handle takes the stream kernel, as the no-alloc entry does, whatever the shape."""
+    h = aio.aio_linear_create(K, N, wt_c, M, flags | aio.AIO_FLAG_STREAM_KERNEL)
     raw = _dev(W)
     sd = _dev(s) if s is not None else None
     sp = sd.data_ptr() if sd is not None else None
