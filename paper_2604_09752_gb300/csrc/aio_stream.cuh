@@ -1009,8 +1009,8 @@ __device__ __forceinline__ void put_x4(uint16_t* xs_row, uint16_t* xg_row, int i
 // silu(t) = t / (1 + e^-t), evaluated with e^-|t| so that the exponential never overflows (for
 // t < 0 it is t e^t / (1 + e^t)).
 __device__ __forceinline__ float silu(float t) {
-    const float e = expf(-fabsf(t));
-    return t >= 0.0f ? t / (1.0f + e) : t * e / (1.0f + e);
+    const float e = __expf(-fabsf(t));
+    return __fdividef(t >= 0.0f ? t : t * e, 1.0f + e);
 }
 
 // x of a projection in a chained decoder step, computed by every thread of the CTA into the staged

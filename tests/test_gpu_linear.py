@@ -105,6 +105,28 @@ def test_linear_parity(aio, wt, K, N, M, layout_):
     lin.close()
 
 
+@pytest.mark.parametrize("wt,K", [("bf16", 2048), ("bf16", 2064), ("int8", 6144), ("int8", 6160)])
+@pytest.mark.parametrize("N", [4864, 4865])
+def test_small_launch_limits(aio, wt, K, N):
+    """At and just past the small-projection launch's limits: 2 x 152 row groups (N = 4864) and
+    96 KB of weights per CTA (bf16 K = 2048, int8 K = 6144, one tile per warp more past them).
+    Inside, one CTA per row group; outside, the stream kernel; both meet the bar at M = 8."""
+    M = 8
+    x, W, s = make_inputs(K, N, M, wt, tag=13)
+    lin = Linear(aio, W, s, max_M=8)
+    want = small_grid(K, N, wt)
+    inside = N == 4864 and K in (2048, 6144)
+    assert (want is not None) == inside
+    assert aio.aio_linear_launch_info(lin.h)["grid"] == (want if inside else n_sms())
+    y = torch.full((M * N,), float("nan"), dtype=torch.float32, device="cuda")
+    lin.run(dev(x), M, y)
+    torch.cuda.synchronize()
+    assert aio.aio_linear_check(lin.h) == 0
+    y_ref, mag = parity.reference(x, W, s)
+    parity.check(y.cpu().numpy().reshape(M, N), y_ref, mag, K, f"limits {wt} K={K} N={N}")
+    lin.close()
+
+
 @pytest.mark.parametrize("wt", ["bf16", "int8"])
 @pytest.mark.parametrize("K,N", [(16, 1), (272, 9), (1040, 37), (4096, 20), (11008, 17)])
 def test_pack_matches_oracle_layout_and_unpacks(aio, wt, K, N):
