@@ -54,7 +54,7 @@ __global__ void __launch_bounds__(kThreads, 2) aio_small_kernel(const __grid_con
     griddep_wait();
 
     const Proj P = load_proj<false>(&D, MT);
-    const I8Consts kc = i8_consts();
+    [[maybe_unused]] const I8Consts kc = i8_consts();
     float d[4][4] = {};
     bool ok = true;
     if (any) {
@@ -62,12 +62,16 @@ __global__ void __launch_bounds__(kThreads, 2) aio_small_kernel(const __grid_con
         if (ok) {
             const int tok = lane >> 2, xtok = min(tok, MT - 1);
             const uint16_t* xrow = P.x + static_cast<size_t>(tok) * K;                             // ragged tiles
-            const uint16_t* xlane = P.x + static_cast<size_t>(xtok) * K + 8 * (lane & 3);        // full tiles
+            [[maybe_unused]] const uint16_t* xlane = P.x + static_cast<size_t>(xtok) * K + 8 * (lane & 3);   // full tiles
             const uint8_t* tp = wbuf;
             for (int kt = kt0; kt < kt1; ++kt) {
                 const int klen = min(kKT, K - kt * kKT);
                 if (rows == kRows && klen == kKT) {
+#if AIO_FFMA
+                    ffma_full_g<I8, MT>(d, tp + lane * 16, P.x + 8 * (lane & 3) + kt * kKT, K);
+#else
                     tile_mma_full<I8>(d, tp + lane * 16, xlane + kt * kKT, kc);
+#endif
                 } else {
                     tile_mma<I8>(d, tp, rows, klen, kt * kKT, lane, P, xrow, kc);
                 }
@@ -79,11 +83,18 @@ __global__ void __launch_bounds__(kThreads, 2) aio_small_kernel(const __grid_con
         }
     }
     // lane (r, c) holds D[row r + 8 (i / 2)][token 2c + i % 2] in sum[i]
+    float sum[4];
+#if AIO_FFMA
+    ffma_finish<MT>(d, sum, lane);
+#else
+#pragma unroll
+    for (int i = 0; i < 4; ++i) sum[i] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
+#endif
     const int gr = lane >> 2, m0 = 2 * (lane & 3);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int m = m0 + (i & 1), r = gr + 8 * (i >> 1);
-        if (m < MT) red[(warp * MT + m) * kRows + r] = (d[0][i] + d[1][i]) + (d[2][i] + d[3][i]);
+        if (m < MT) red[(warp * MT + m) * kRows + r] = sum[i];
     }
     __syncthreads();
     const int t = threadIdx.x;
