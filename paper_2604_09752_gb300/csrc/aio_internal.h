@@ -38,14 +38,21 @@
 #ifndef AIO_SLOT_KB_I8
 #define AIO_SLOT_KB_I8 AIO_SLOT_KB   // the same for int8 weights (4 KB tiles)
 #endif
-// Launches with M >= AIO_WIDE_M token rows use a ring of AIO_RING_KB_WIDE per warp instead, so that
-// the area left for staged x holds M rows of the 4096-column projections (and M <= 4 rows of
-// K = 11008 would fit it too): at such widths a tile's x read from L2 costs more than a ring slot.
+// Plain launches with M >= AIO_WIDE_M token rows (int8 weights: M >= AIO_WIDE_M_I8) use a ring of
+// AIO_RING_KB_WIDE per warp instead, so that the area left for staged x holds M rows of the
+// 4096-column projections (and M <= 4 rows of K = 11008): at such widths a tile's x read from L2
+// costs more than a ring slot.  Such launches refill a slot as soon as its tiles are in registers,
+// so two slots keep as many copies in flight as three did.  int8 tiles take longer to compute per
+// byte, which is why they gain from the wide layout from two rows up.  The chained kernels always use
+// the narrow layout.
 #ifndef AIO_RING_KB_WIDE
 #define AIO_RING_KB_WIDE 16
 #endif
 #ifndef AIO_WIDE_M
 #define AIO_WIDE_M 5
+#endif
+#ifndef AIO_WIDE_M_I8
+#define AIO_WIDE_M_I8 2
 #endif
 
 namespace aio {
@@ -77,10 +84,13 @@ struct SmemLayout {
     static_assert(kSlotBytesI8 % 4096 == 0 && kStagesI8 >= 2, "a slot holds whole tiles; a ring has >= 2 slots");
     static_assert(kXsOffset % 16 == 0 && kXsBytes > 0, "ring does not fit in shared memory");
 };
-using NarrowLayout = SmemLayout<AIO_RING_KB>;       // launches of M < AIO_WIDE_M token rows
-using WideLayout = SmemLayout<AIO_RING_KB_WIDE>;    // M >= AIO_WIDE_M
-template <int MT>
-using LayoutFor = SmemLayout<(MT >= AIO_WIDE_M ? AIO_RING_KB_WIDE : AIO_RING_KB)>;
+using NarrowLayout = SmemLayout<AIO_RING_KB>;       // launches of fewer token rows, and every chained launch
+using WideLayout = SmemLayout<AIO_RING_KB_WIDE>;    // plain launches of M >= AIO_WIDE_M (int8: AIO_WIDE_M_I8)
+// The layout of a launch of MT token rows, int8 or bf16 weights, chained or plain.
+template <int MT, bool I8, bool CH>
+constexpr bool kWideLaunch = !CH && MT >= (I8 ? AIO_WIDE_M_I8 : AIO_WIDE_M);
+template <int MT, bool I8, bool CH>
+using LayoutFor = SmemLayout<(kWideLaunch<MT, I8, CH> ? AIO_RING_KB_WIDE : AIO_RING_KB)>;
 // The narrow layout's values, for code that runs at every width (the read probe, attention) and for
 // the chained step, whose kernels exist for M <= 4 only.
 constexpr int kRingBytesPerWarp = NarrowLayout::kRingBytes;
@@ -183,7 +193,8 @@ cudaError_t prepare_kernels();  // per-device kernel attributes (dynamic shared 
 // pdl: programmatic dependent launch; coop: cooperative launch (all CTAs co-resident).
 using StreamFn = void (*)(const StreamArgs);
 constexpr int kMaxChainM = 4;   // token rows of a chained step (its kernels are instantiated for M <= 4)
-static_assert(kMaxChainM < AIO_WIDE_M, "the chained step's staging limit is the narrow layout's");
+static_assert(!kWideLaunch<kMaxChainM, true, true> && !kWideLaunch<kMaxChainM, false, true>,
+              "the chained step's staging limit is the narrow layout's");
 static_assert(kAttnMergeScratch <= kXsBytes, "the attention merge's scratch fits the staging area");
 StreamFn chain_stream_fn(bool i8, int M, bool phases);   // aio_chain.cu
 StreamFn chain_phase_stream_fn(bool i8, int M);          // aio_chain_ph.cu

@@ -12,8 +12,9 @@
 //   * Rings.  One CTA per SM; each warp owns a shared-memory ring of slots.  Lane 0 issues one
 //     cp.async.bulk per slot (global -> shared, L2 evict-first) completing on the slot's mbarrier;
 //     the warp waits (bounded by %globaltimer), computes, and refills the slot.  The issue cursor
-//     runs ahead across projection boundaries: weights never depend on x.  Plain launches of
-//     M >= AIO_WIDE_M (two slots per warp) read a slot into registers and refill it before computing.
+//     runs ahead across projection boundaries: weights never depend on x.  The wide launches (two
+//     slots per warp: bf16 M >= 5, int8 M >= 2) read a slot into registers and refill it before
+//     computing.
 //   * x.  Once per CTA and projection, warp 0 stages x into shared memory (one bulk copy per token
 //     row, rows padded by 64 B) when it fits; otherwise the lanes read x from global memory.
 //   * Arithmetic on the tensor cores: mma.sync.m16n8k16, bf16 in, fp32 accumulate, with A = W
@@ -1318,7 +1319,7 @@ template <int MT, bool I8>
 __device__ __noinline__ RingCtx attn_phase(RingCtx r, const StreamArgs& s, const ProjDesc* D, uint8_t* ring,
                                            uint64_t* bars, int z, int lane, uint64_t pol, int p) {
     using TL = TileT<I8>;
-    using SL = LayoutFor<MT>;
+    using SL = LayoutFor<MT, I8, true>;   // phases run in chained kernels
     constexpr int C = TL::kChunk;
     constexpr int S = I8 ? SL::kStagesI8 : SL::kStages;
     const int Z = s.Z;
@@ -1448,7 +1449,7 @@ __device__ __noinline__ RingCtx attn_phase(RingCtx r, const StreamArgs& s, const
 template <int MT, bool I8, bool CH, bool PH = false>
 __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_constant__ StreamArgs s) {
     using TL = TileT<I8>;
-    using SL = LayoutFor<MT>;
+    using SL = LayoutFor<MT, I8, CH>;
     static_assert(CH || !PH, "phases belong to chained steps");
     static_assert(!PH || TL::kSlot >= kAttnSlot, "a ring slot holds one attention unit");
     constexpr int C = TL::kChunk;
@@ -1665,8 +1666,8 @@ __global__ void __launch_bounds__(kThreads, 1) aio_stream_kernel(const __grid_co
                     const int nt = min(C, tend - t);
                     const uint8_t* tp = ring + cslot * TL::kSlot;
 #if !AIO_FFMA
-                    if constexpr (FAST && !CH && MT >= AIO_WIDE_M) {
-                        // Early release (plain launches of M >= AIO_WIDE_M, whose rings have two slots):
+                    if constexpr (FAST && kWideLaunch<MT, I8, CH>) {
+                        // Early release (the wide launches, whose rings have two slots):
                         // read the slot's tiles of W into registers and hand the slot back to the
                         // issuing lane before the arithmetic, so that its next copy is in flight while
                         // these tiles are computed.  Every lane's reads are ordered before lane 0's
