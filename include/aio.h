@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define AIO_ABI_VERSION 7
+#define AIO_ABI_VERSION 8
 
 typedef enum {
     AIO_OK = 0,

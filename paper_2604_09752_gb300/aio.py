@@ -43,7 +43,7 @@ AIO_STEP_PERSISTENT = 0x4
 AIO_ROWS_PER_GROUP = 16
 AIO_K_TILE = 256
 AIO_NOALLOC_SCRATCH_BYTES = 1048576
-AIO_ABI_VERSION = 7
+AIO_ABI_VERSION = 8
 AIO_X_GIVEN = 0
 AIO_X_RMSNORM = 1
 AIO_X_SWIGLU = 2
@@ -113,6 +113,9 @@ for _f, (_res, _args) in _SIGS.items():
     _fn = getattr(_lib, _f)
     _fn.restype = _res
     _fn.argtypes = _args
+if _lib.aio_abi_version() != AIO_ABI_VERSION:
+    raise ImportError(f"{LIB_PATH} has ABI version {_lib.aio_abi_version()}, the binding expects "
+                      f"{AIO_ABI_VERSION}: rebuild it (paper_2604_09752_gb300.build)")
 
 
 def lib():

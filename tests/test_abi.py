@@ -46,7 +46,7 @@ def test_no_torch_types_in_signatures():
 
 
 def test_abi_version_and_status_strings(aio):
-    assert aio.aio_abi_version() == 7
+    assert aio.aio_abi_version() == aio.AIO_ABI_VERSION == 8
     for code in range(8):
         assert aio.aio_status_string(code).startswith("AIO_")
     assert aio.aio_status_string(99) == "AIO_ERR_UNKNOWN"
