@@ -473,8 +473,9 @@ def bench_pld_ops(args):
 
 
 def configs_block(args, peak, local, main_rec):
-    """Every BASELINE config in one object (configs 1 to 5), then the later rows of the path (chained
-    step, decode attention, PLD drafting and acceptance), with the clocks seen meanwhile."""
+    """Every named workload in one object (the single 2048 x 2048 layer, the 1B and 7B bf16 steps, the
+    7B int8 step and the PLD widths), then the later rows of the path (chained step, decode
+    attention, PLD drafting and acceptance), with the clocks seen meanwhile."""
     from synth import workloads as swl
     clocks = ClockSampler(local)
     t0 = time.time()
@@ -676,7 +677,7 @@ def main():
                     help="repeat oracle passes over the row sample for at least this long")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--configs", choices=["all", "baseline", "none"], default="all",
-                    help="the configs block (N = 1 only): every BASELINE config (baseline), plus the chained step, "
+                    help="the configs block (N = 1 only): every named workload (baseline), plus the chained step, "
                          "decode attention and PLD drafting (all), or nothing (none)")
     ap.add_argument("--step-mode", choices=["persistent", "chain"], default="persistent",
                     help="one cooperative launch per step (default) or one launch per projection")
